@@ -1,0 +1,487 @@
+#!/usr/bin/env python
+"""Benchmark of the BaryCache skipped-step forecast on GB300.
+
+One step = one skipped diffusion step of the workload: the host weight solve (Diff Key memo,
+Eqs. 8-12) plus the grouped forecast kernel over every cached layer (Eq. 13), issued through
+the C ABI on a torch stream.  Inputs (the K history slots) are resident in HBM before the
+timed region and are far larger than L2 (so no L2 flush is needed).  Steps alternate between
+the skipped steps that share one history window, as in the equal-spaced schedule.
+
+Prints one JSON line (rank 0).  Default workload: the video DiT (60 x [1, 118800, 3072] bf16,
+K = 3; 131 GB of cache, 175 GB of HBM traffic per step).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload t2v|mmdit-t2i|t2i-1024|c2i-512|c2i-256] [--K 3] [--sweep]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "forecast HBM GB/s and % of GB300 peak; forecast elems/s; cache VRAM bytes"
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="t2v")
+    ap.add_argument("--K", type=int, default=None)
+    ap.add_argument("--sweep", action="store_true", help="also time every K of the workload")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------------------- helpers
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            return float(json.load(fh)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("bc_forecast.cu", "bc_internal.h"):
+        with open(os.path.join(ROOT, "paper_2608_28670_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str, K: int):
+    """DRAM bytes per launch of the forecast kernel from the committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "forecast_kernel_traffic.json.txt")
+    try:
+        with open(path) as fh:
+            rec = json.loads(fh.read().split("\n", 1)[1])  # first line is a comment
+    except Exception:
+        return None
+    if rec.get("kernel_source_sha256_16") != kernel_source_hash():
+        return None
+    per_elem = rec.get("dram_bytes_per_output_element", {}).get(f"K{K}")
+    return per_elem
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) during the timed region."""
+
+    def __init__(self, enabled: bool):
+        self.proc = None
+        self.path = None
+        if not enabled:
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        try:
+            idx = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[0] or "0"
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", idx, f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        with open(self.path) as fh:
+            for line in fh:
+                f = [x.strip() for x in line.split(",")]
+                if len(f) >= 7:
+                    try:
+                        rows.append((float(f[0]), float(f[1]), float(f[2]), f[3:7]))
+                    except ValueError:
+                        pass
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[3]) if v == "Active"})
+        loaded = [r for r in rows if r[2] > 300.0] or rows
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows), "samples_under_load": len(loaded),
+                "power_w_max": max(r[2] for r in rows)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def window_targets(w, K):
+    rep = w.representative(K)
+    ts = [p.t for p in w.problems(K) if p.node_steps == rep.node_steps]
+    return ts or [rep.t]
+
+
+def time_forecast(run, steps, warmup, stream, dist=None):
+    import torch
+    ts = window_targets(run.w, run.K)
+    for i in range(warmup):
+        run.forecast(ts[i % len(ts)])
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    launches0 = run.stats()["kernel_launches"]
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    torch.cuda.synchronize()
+    for i in range(steps):
+        starts[i].record()
+        run.forecast(ts[i % len(ts)])
+        ends[i].record()
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    per_step = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    launches = run.stats()["kernel_launches"] - launches0
+    return total_ms, per_step, launches
+
+
+def run_ours(args):
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    from paper_2608_28670_gb300.configs import WORKLOADS, T2V_HBM_BUDGET
+    from paper_2608_28670_gb300.runner import WorkloadRun
+    import __graft_entry__
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+        torch.cuda.set_device(local)
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist = tdist
+    else:
+        torch.cuda.set_device(0)
+    __graft_entry__.build_libraries()   # no-op when the libraries are current
+    w = WORKLOADS[args.workload]
+    K = args.K or w.K
+    budget = T2V_HBM_BUDGET if w.name == "t2v" else None
+    stream = torch.cuda.current_stream().cuda_stream
+
+    run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
+    try:
+        torch.cuda.synchronize()
+        clocks = ClockSampler(not args.no_clocks)
+        total_ms, per_step, launches = time_forecast(run, args.steps, args.warmup, stream, dist)
+        clk = clocks.stop()
+        ms = total_ms / args.steps
+        if dist is not None:
+            t = torch.tensor([ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        alg = run.algorithmic_bytes()
+        value = alg * world / (ms * 1e-3) / 1e9
+        elems = run.w.layer_numel * run.n_feat + (run.numels[-1] if run.euler else 0)
+        launches_per_step = launches / args.steps
+        kernel_ms = statistics.mean(per_step) / max(launches_per_step, 1)
+        per_launch_bytes = alg / max(launches_per_step, 1)
+        peak, peak_kind = measured_peak()
+        achieved = per_launch_bytes / (kernel_ms * 1e-3) / 1e9
+        traffic_per_elem = profiled_traffic(w.name, K)
+        per_launch_elems = elems / max(launches_per_step, 1)
+        result = {
+            "metric": METRIC, "value": round(value, 1), "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {
+                "workload": w.name,
+                "layers": f"{w.n_layers}x{list(w.layer_shape)}"
+                          + (f" + euler {list(w.euler_shape)}" if w.euler_shape else ""),
+                "storage_dtype": "bf16" if w.dtype == bc.DTYPE_BF16 else "f32",
+                "K": K, "forecast_calls_per_step": run.calls,
+                "layers_per_call": run.window,
+                "weights": "paper Eqs. 8-12, delta_H table, lambda 0, C 10, eta 1e-12",
+                "targets": window_targets(w, K), "nodes": list(run.problem.nodes),
+                "l2": "inputs larger than L2 (no flush)",
+                "parallelism": f"replicas x{world}",
+            },
+            "pct_of_measured_peak": round(100 * value / world / peak, 2),
+            "pct_of_nominal_8tbs": round(100 * value / world / NOMINAL_HBM_GBS, 2),
+            "elems_per_s": round(elems * world / (ms * 1e-3), 1),
+            "per_skipped_step_ms": round(ms, 4),
+            "cache_bytes": bc.bc_cache_bytes(run.h),
+            "algorithmic_bytes_per_step": alg,
+            "roofline": {
+                "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+                "traffic": (round(traffic_per_elem * per_launch_elems)
+                            if traffic_per_elem else None),
+                "kernel": "bc::forecast_kernel", "avg_launch_ms": round(kernel_ms, 4),
+                "algorithmic_bytes_per_launch": per_launch_bytes,
+            },
+            "gpu_launches": launches,
+        }
+        if clk:
+            result["clocks"] = clk
+        if args.sweep and w.K_sweep:
+            sweep = {}
+            run.close()
+            run = None
+            torch.cuda.empty_cache()
+            for k in w.K_sweep:
+                r = WorkloadRun(w, K=k, budget_bytes=budget, stream=stream)
+                try:
+                    tm, ps, ln = time_forecast(r, args.steps, args.warmup, stream, dist)
+                    a = r.algorithmic_bytes()
+                    m = tm / args.steps
+                    sweep[f"K{k}"] = {"GB/s": round(a / (m * 1e-3) / 1e9, 1), "ms": round(m, 4),
+                                      "cache_bytes": bc.bc_cache_bytes(r.h),
+                                      "calls_per_step": r.calls, "layers_per_call": r.window,
+                                      "launches": ln}
+                finally:
+                    r.close()
+                    torch.cuda.empty_cache()
+            result["sweep"] = sweep
+            run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
+        if not args.no_e2e:
+            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
+        if rank == 0 and world == 1 and not args.no_cpu_baseline:
+            result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
+    finally:
+        if run is not None:
+            run.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+def _continuation(run, i):
+    """(time of the i-th next full step, the skipped step after it) continuing the window's
+    spacing."""
+    p = run.problem
+    nodes = p.nodes
+    step = (nodes[0] - nodes[1]) if len(nodes) > 1 else 2.0 * (p.t - nodes[0])
+    off = p.t - nodes[0]
+    t_full = nodes[0] + (i + 1) * step
+    return t_full, t_full + off
+
+
+def e2e(run, steps, world, dist):
+    """Same metric through the public API with host buffers.  Per step: the new full-step
+    features (one slot, every layer) are copied from pinned host memory into the next cache
+    slot and committed (zero-copy push, Eq. 6), the following skipped step is forecast, and
+    the forecast is read back into pinned host memory.  One pinned host buffer of one slot
+    serves both directions (the read-back of step i is the input of step i + 1)."""
+    import numpy as np
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    from paper_2608_28670_gb300.runner import device_view
+
+    eb = run.w.elem_bytes
+    ob = 2 if run.out_dtype == bc.DTYPE_BF16 else 4
+    sizes = [n * eb for n in run.numels]
+    offs = np.cumsum([0] + sizes)
+    total = int(offs[-1])
+    host = np.empty(total, dtype=np.uint8)
+    cudart = torch.cuda.cudart()
+    rc = cudart.cudaHostRegister(host.ctypes.data, total, 0)
+    if int(rc) != 0:
+        return {"unavailable": f"cudaHostRegister of {total} bytes failed ({rc})"}
+    try:
+        tdt = torch.bfloat16 if run.w.dtype == bc.DTYPE_BF16 else torch.float32
+        hviews = [torch.from_numpy(host[offs[l]:offs[l + 1]]).view(tdt)
+                  for l in range(len(run.numels))]
+        # initial content: the current newest slot (a real full-step feature)
+        newest = bc.bc_cache_slot_ptrs(run.h, 0, len(run.numels))
+        for l, n in enumerate(run.numels):
+            hviews[l].copy_(device_view(newest[l], n, run.w.dtype).view(tdt))
+        torch.cuda.synchronize()
+
+        def one_step(i):
+            t_full, t_target = _continuation(run, i)
+            slots = bc.bc_cache_next_slot_ptrs(run.h, len(run.numels))
+            for l, n in enumerate(run.numels):
+                device_view(slots[l], n, run.w.dtype).view(tdt).copy_(hviews[l], non_blocking=True)
+            bc.bc_cache_commit(run.h, t_full)
+            for c in range(run.calls):
+                run.forecast_call(c, t_target)
+                for k in range(run.window):
+                    l = c * run.window + k
+                    if l < run.n_feat:
+                        hviews[l].copy_(run.outs[k].view(tdt) if ob == eb else run.outs[k],
+                                        non_blocking=True)
+
+        one_step(0)                      # warm-up
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        t0 = time.perf_counter()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for i in range(steps):
+            one_step(i + 1)
+        b.record()
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        ms = a.elapsed_time(b) / steps
+        if dist is not None:
+            t = torch.tensor([ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        alg = run.algorithmic_bytes()
+        return {"value": round(alg * world / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                "h2d_bytes_per_step": total, "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
+                "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
+                "path": "pinned host -> next cache slot (bc_cache_next_slot_ptrs + "
+                        "bc_cache_commit) -> bc_forecast -> pinned host"}
+    finally:
+        cudart.cudaHostUnregister(host.ctypes.data)
+
+
+CHUNK = 1 << 22   # elements per oracle call in the CPU samples
+
+
+def _time_oracle(chunks, W, seconds):
+    """Time the oracle over host chunks (list of lists of K arrays) until `seconds` pass or
+    the chunks run out; returns (elements, seconds)."""
+    import oracle
+    done, spent = 0, 0.0
+    for F in chunks:
+        t0 = time.perf_counter()
+        oracle.combine(F, W)
+        spent += time.perf_counter() - t0
+        done += F[0].size
+        if spent >= seconds:
+            break
+    return done, spent
+
+
+def cpu_baseline_from_device(run, seconds):
+    """The fp64 oracle, single-threaded on the host, over a bounded sample of the same
+    workload: chunks of 4 Mi elements of the live history slots (copied to the host first,
+    outside the timed region), layers round-robin."""
+    import numpy as np
+    import oracle
+    from paper_2608_28670_gb300.runner import device_view
+
+    p = run.problem
+    W = oracle.paper_weights(list(p.nodes), p.t)
+    m = len(p.nodes)
+    slots = [bc_slot_ptrs(run, j) for j in range(m)]
+
+    def chunk(c):
+        l = c % run.n_feat
+        n = run.numels[l]
+        size = min(CHUNK, n)
+        off = ((c * 2654435761) % max(1, n - size + 1)) // 8 * 8
+        F = []
+        for j in range(m):
+            v = device_view(slots[j][l], n, run.w.dtype)[off:off + size].cpu().numpy()
+            F.append(v.view(np.uint16) if v.dtype == np.int16 else v)
+        return F
+
+    first = chunk(0)
+    n1, t1 = _time_oracle([first], W, 1e9)
+    want = max(1, min(400, int(seconds / max(t1, 1e-6))))
+    chunks = [chunk(c) for c in range(1, want)]
+    n2, t2 = _time_oracle(chunks, W, seconds)
+    elems, secs = n1 + n2, t1 + t2
+    per_elem = run.algorithmic_bytes() / (run.w.layer_numel * run.n_feat)
+    return {"value": round(elems * per_elem / secs / 1e9, 4), "unit": "GB/s", "cores": 1,
+            "kind": "oracle",
+            "elems_per_s": round(elems / secs, 1),
+            "sample": f"{elems} elements ({len(chunks) + 1} chunks of <= {CHUNK} consecutive "
+                      f"elements, layers round-robin) of the K={m} history slots, fp64 oracle, "
+                      f"{secs:.1f} s"}
+
+
+def bc_slot_ptrs(run, j):
+    from paper_2608_28670_gb300 import barycache as bc
+    return bc.bc_cache_slot_ptrs(run.h, j, len(run.numels))
+
+
+def run_reference(args):
+    """The oracle as the reference arm: fp64, single-threaded, on the host cores, on a
+    bounded host-generated sample of the same workload per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    import oracle
+    from paper_2608_28670_gb300 import synth
+    from paper_2608_28670_gb300.configs import WORKLOADS
+    oracle.build()
+    w = WORKLOADS[args.workload]
+    K = args.K or w.K
+    p = w.representative(K)
+    n = 1 << 25                       # 32 Mi elements per node: inputs larger than the host L3
+    nodes_oldest_first = list(reversed(p.nodes))
+    feats = synth.host_trajectories([(n,)], [w.tau(t) for t in nodes_oldest_first],
+                                    dtype="bf16" if w.elem_bytes == 2 else "f32",
+                                    degree=w.degree, noise_std=w.noise_std, seed=2026)
+    F = [f[0] for f in reversed(feats)]        # newest first
+    W = oracle.paper_weights(list(p.nodes), p.t)
+    per_elem = (K * w.elem_bytes + w.elem_bytes)
+    reps = 1
+    for _ in range(args.warmup):
+        for _ in range(reps):
+            oracle.combine(F, W)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            oracle.combine(F, W)
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * sum(times) / len(times)
+    value = reps * n * per_elem / (ms * 1e-3) / 1e9
+    sample = f"{reps} x {n} elements per step of one [{n}] bf16 slice at K={K}, fp64 oracle"
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": w.name, "K": K, "nodes": list(p.nodes), "target": p.t,
+                      "sample_elements_per_step": reps * n},
+           "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1,
+                            "kind": "oracle", "sample": sample},
+           "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

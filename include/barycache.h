@@ -1,0 +1,198 @@
+/*
+ * barycache.h -- C ABI of the GB300 (sm_103a) BaryCache skipped-step forecast library.
+ *
+ * BaryCache (Barycentric Extrapolator, Sec. 3.2-3.3) accelerates DiT sampling by running
+ * the full model only on some diffusion steps ("full steps") and predicting the cached
+ * features on the others ("skipped steps" / cache forward) as a fixed linear combination
+ * of the H most recent full-step features:
+ *
+ *     x_hat_t = W_i H^T = sum_{j=1..H} W_j x_{f=-j}                           (Eq. 13)
+ *
+ * The weights W depend only on the timestep differences t - s_j and the hyper-parameters
+ * (the "online decoupling" of Sec. 1 and the Diff Key of Eq. 7), so they are solved on
+ * the host in fp64 and memoised; the weight application streams every cached byte once
+ * through one persistent CUDA kernel.
+ *
+ * Conventions shared by every call:
+ *  - Node j = 1 (C index 0) is the most recent cached feature x_{f=-1}; nodes are listed
+ *    newest first everywhere (Sec. 3.2, "Get Key").
+ *  - "Layer" is one cached tensor (a block output, or the stepwise feature of Eq. 5),
+ *    treated as a flat contiguous vector of `numel` elements.
+ *  - Device pointers are plain CUDA device addresses on the device that was current when
+ *    the cache was created.  Every device pointer passed in must be 16-byte aligned
+ *    (BC_ERR_ALIGNMENT otherwise) and must hold the stated number of elements (the
+ *    library cannot check sizes of foreign allocations).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  All
+ *    device work is enqueued on it asynchronously; errors are reported by return value
+ *    only, and no call blocks on the device except bc_cache_create/destroy.
+ *  - Host-side cache state (ring head, node times) changes when the call is made, so
+ *    pushes and forecasts on one handle must be issued from one thread, in order, on one
+ *    stream (or with the caller's own synchronisation).
+ *  - No exception crosses the ABI; device code never traps or waits.
+ */
+#ifndef BARYCACHE_H
+#define BARYCACHE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Largest history length H (the paper ablates H = 2, 3, 4: Sec. 4.4). */
+#define BC_MAX_K 4
+
+typedef enum {
+    BC_OK = 0,
+    BC_ERR_INVALID_ARG = 1,        /* bad size, count, dtype, mode, null pointer, overlap */
+    BC_ERR_ALIGNMENT = 2,          /* a device pointer is not 16-byte aligned */
+    BC_ERR_OOM = 3,                /* device allocation failed (cache arena) */
+    BC_ERR_CUDA = 4,               /* a CUDA runtime call failed; see bc_last_error() */
+    BC_ERR_NOT_READY = 5,          /* forecast before any feature was pushed */
+    BC_ERR_DUPLICATE_NODE = 6,     /* pushed t equals a timestep already in the window */
+    BC_ERR_DEGENERATE_WEIGHTS = 7, /* Eq. 11 normaliser vanishes; run a full step instead */
+    BC_ERR_BAD_HANDLE = 8          /* null, destroyed or foreign handle */
+} bc_status;
+
+typedef enum { BC_DTYPE_F32 = 0, BC_DTYPE_BF16 = 1 } bc_dtype;
+
+/* Weight construction.
+ *  BC_MODE_EXACT: the polynomial extrapolant through the live nodes, in barycentric form:
+ *      c_j = (w_j / (t - s_j)) / sum_k (w_k / (t - s_k)),  w_j = 1 / prod_{k!=j} (s_j - s_k),
+ *      and c = e_j exactly when t == s_j (Sec. 1: barycentric interpolation as a
+ *      reformulation of polynomial interpolation).
+ *  BC_MODE_PAPER: the stabilised weights of Eqs. 8-12 (trapezoid node factors, raw weight
+ *      u_j = c_j (-1)^j / (t - s_j), clip to [-C, C], signed decay power with eta, and the
+ *      blend lambda towards x_{f=-1}). */
+typedef enum { BC_MODE_EXACT = 0, BC_MODE_PAPER = 1 } bc_mode;
+
+typedef struct {
+    int32_t mode;   /* bc_mode */
+    double delta;   /* decay power of Eq. 11; <= 0 selects delta_H by the live window size
+                       H: 1.0 (H <= 2), 0.95 (H = 3), 0.7 (H = 4) (Sec. 3.2, under Eq. 10) */
+    double lambda;  /* Eq. 12 blend in [0, 1]: W = (1 - lambda) alpha + lambda e_1 */
+    double clip_C;  /* Eq. 10 clip, > 0 (paper: 10) */
+    double eta;     /* Eq. 11 offset, >= 0 (paper: 1e-12) */
+} bc_params;
+
+typedef struct bc_cache *bc_handle;
+
+typedef struct {
+    int64_t forecasts;       /* successful bc_forecast / bc_forecast_step calls */
+    int64_t pushes;          /* successful bc_cache_push / bc_cache_commit calls */
+    int64_t kernel_launches; /* CUDA kernels this handle has launched */
+    int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
+    int64_t memo_misses;     /* Diff Key lookups that ran the solver */
+} bc_stats;
+
+/* ---------------------------------------------------------------- host-only calls */
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int bc_version(void);
+
+/* Static description of a status code.  Never NULL. */
+const char *bc_status_string(bc_status s);
+
+/* Detail message of the most recent failing call made by this thread ("" if none).
+ * The string stays valid until this thread's next library call. */
+const char *bc_last_error(void);
+
+/* Fill `p` with the paper's defaults: PAPER mode, delta by table, lambda 0, C 10,
+ * eta 1e-12 (Sec. 3.2; lambda = 0 for C2I/T2I, Sec. 4.1). */
+void bc_params_default(bc_params *p);
+
+/* Weight construction (Eqs. 8-12, or the exact barycentric form) for `m` nodes
+ * `nodes[0..m-1]` (newest first) and target `t`, in fp64, into c_out[0..m-1].
+ * p == NULL uses bc_params_default.  Pure host arithmetic: needs no GPU.
+ * Errors: INVALID_ARG (m outside 1..BC_MAX_K, bad params, NaN input),
+ * DUPLICATE_NODE (EXACT mode with two equal nodes), DEGENERATE_WEIGHTS. */
+bc_status bc_solve(const double *nodes, int m, double t, const bc_params *p, double *c_out);
+
+/* Device bytes a cache of these layers would hold: K slots, each holding every layer at a
+ * 256-byte aligned offset (the memory claim of Sec. 1 / Fig. 1: a stepwise cache stores H
+ * feature copies, not N x Q).  Needs no GPU. */
+bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
+                             int64_t *bytes);
+
+/* ------------------------------------------------------------ cache lifecycle */
+
+/* Create the cache context H_t of Eq. 6 for `n_layers` tensors of numels[l] elements of
+ * `dtype`, with history length K (1..BC_MAX_K).  Allocates one device arena of
+ * bc_cache_bytes_for(...) bytes on the current device (the only device allocation the
+ * library makes; freed by bc_cache_destroy).  p == NULL uses the paper's defaults.
+ * Blocks until the allocation is done.  Errors: INVALID_ARG, OOM, CUDA. */
+bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
+                          const bc_params *p, bc_handle *out);
+
+/* Free the arena (synchronises the device first so no enqueued work still reads it). */
+bc_status bc_cache_destroy(bc_handle h);
+
+/* Device bytes held by this cache (arena only; host bookkeeping is not counted). */
+bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
+
+/* Replace the weight parameters (clears the weight memo). */
+bc_status bc_cache_set_params(bc_handle h, const bc_params *p);
+
+/* Forget every pushed node (the arena keeps its bytes; nothing is enqueued). */
+bc_status bc_cache_reset(bc_handle h);
+
+/* Insert a full-step feature (Eq. 6): the oldest slot is evicted by rotating the ring
+ * head, and layer_ptrs[l] (device, numels[l] elements of the cache dtype, 16-byte
+ * aligned) is copied into it by one grouped copy kernel on `stream`.  `t` is the
+ * timestep of this full step.  Errors: INVALID_ARG (null pointer, non-finite t, source
+ * overlapping the arena), ALIGNMENT, DUPLICATE_NODE (t equals a node that stays in the
+ * window), CUDA. */
+bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, void *stream);
+
+/* Zero-copy push, part 1: the device addresses (one per layer) of the slot the next push
+ * will fill.  The caller (e.g. the DiT writing its block outputs) writes the new feature
+ * there, then calls bc_cache_commit.  When the window is full this slot still holds the
+ * oldest node, so no forecast may be enqueued between the first write and the commit. */
+bc_status bc_cache_next_slot_ptrs(bc_handle h, void **out_ptrs);
+
+/* Zero-copy push, part 2: make the slot returned by bc_cache_next_slot_ptrs the newest
+ * node, with timestep t.  No device work.  Errors as bc_cache_push. */
+bc_status bc_cache_commit(bc_handle h, double t);
+
+/* Live node timesteps, newest first, into nodes_out[0..*m_out-1] (capacity BC_MAX_K). */
+bc_status bc_cache_nodes(bc_handle h, double *nodes_out, int *m_out);
+
+/* Device addresses of node j's stored tensors (j = 0 is x_{f=-1}); j < live count. */
+bc_status bc_cache_slot_ptrs(bc_handle h, int j, void **out_ptrs);
+
+/* The weights a forecast at t_new would use (fp64, before rounding to fp32), newest
+ * first, m_out = number of live nodes used.  Goes through the Diff Key memo. */
+bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
+
+/* ------------------------------------------------------------ the forecast (Eq. 13) */
+
+/* Skipped-step forecast: for every layer l with out_ptrs[l] != NULL,
+ *     out_l[e] = sum_{j=1..m} W_j * F_{l,j}[e],   m = min(pushed, K),
+ * with W from the solver (memoised by Diff Key, rounded to fp32), fp32 accumulation in
+ * node order j = 1..m, and the result stored as `out_dtype` (bf16: round to nearest even).
+ * One persistent grouped kernel launch covers every selected layer (more only for
+ * caches of several hundred layers).  Layers with a NULL output are skipped, which also
+ * serves to forecast a window of layers.  Outputs must not overlap the arena.
+ * Errors: INVALID_ARG, ALIGNMENT, NOT_READY, DEGENERATE_WEIGHTS, CUDA. */
+bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
+                      void *stream);
+
+/* Forecast fused with one explicit Euler step of the flow-matching sampler (Sec. 4.1:
+ * Euler sampling for T2V).  Layer `v_layer` holds the cached model output (velocity):
+ *     v_hat[e] = sum_j W_j V_j[e],    x[e] <- x[e] + dt * v_hat[e]   (fp32 math)
+ * in the same launch as the forecast of every other layer with a non-NULL out_ptrs[l].
+ * x (device, numels[v_layer] elements of x_dtype, updated in place) must not alias any
+ * output.  out_ptrs[v_layer] may be NULL (v_hat not stored) or receive v_hat.
+ * dt = t_next - t_new (negative when t runs from 1 to 0).  Errors as bc_forecast. */
+bc_status bc_forecast_step(bc_handle h, double t_new, double dt, void *const *out_ptrs,
+                           bc_dtype out_dtype, int v_layer, void *x, bc_dtype x_dtype,
+                           void *stream);
+
+/* Counters of this handle (see bc_stats). */
+bc_status bc_cache_stats(bc_handle h, bc_stats *out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BARYCACHE_H */

@@ -1,0 +1,651 @@
+// bc_host.cpp -- host side of the BaryCache forecast library: the fp64 weight solver,
+// the Diff Key memo, the ring-buffer cache context and the C ABI (include/barycache.h).
+//
+// Paper: BaryCache, Sec. 3.2 (cache context, Eq. 6; Diff Key, Eq. 7; weights, Eqs. 8-12)
+// and Sec. 3.3 (full step stores the feature, cache forward applies Eq. 13).
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <new>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+#include "barycache.h"
+#include "bc_internal.h"
+
+namespace {
+
+thread_local std::string t_last_error;
+
+bc_status fail(bc_status s, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+bc_status fail(bc_status s, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_last_error = buf;
+    return s;
+}
+
+bc_status cuda_fail(int err, const char *what) {
+    return fail(BC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(static_cast<cudaError_t>(err)));
+}
+
+// ------------------------------------------------------------------ weight solver
+//
+// Both modes are evaluated from the differences d_j = t - s_j only, so that a memo entry
+// keyed by the differences returns exactly what a fresh solve would (Eq. 7: the weights
+// depend on the schedule through t - s_j alone).
+
+// delta_H of Sec. 3.2 (text between Eqs. 10 and 11); a single node normalises to 1 for
+// any delta.
+double delta_for_window(int H) {
+    if (H <= 2) return 1.0;
+    if (H == 3) return 0.95;
+    return 0.7;
+}
+
+bool params_valid(const bc_params &p) {
+    if (p.mode != BC_MODE_EXACT && p.mode != BC_MODE_PAPER) return false;
+    if (!std::isfinite(p.delta) || !std::isfinite(p.lambda)) return false;
+    if (!(p.clip_C > 0.0) || !(p.eta >= 0.0) || !std::isfinite(p.eta)) return false;
+    if (p.lambda < 0.0 || p.lambda > 1.0) return false;
+    return true;
+}
+
+// Exact polynomial extrapolation, barycentric form:
+//   c_j = (w_j / d_j) / sum_k (w_k / d_k),  w_j = 1 / prod_{k!=j} (s_j - s_k),
+// with s_j - s_k = d_k - d_j.  A node hit (d_j == 0) is the interpolation property e_j.
+bc_status solve_exact(const double *d, int m, double *c) {
+    for (int j = 0; j < m; ++j)
+        for (int k = j + 1; k < m; ++k)
+            if (d[j] == d[k]) return fail(BC_ERR_DUPLICATE_NODE, "two nodes share a timestep");
+    for (int j = 0; j < m; ++j) {
+        if (d[j] == 0.0) {
+            for (int k = 0; k < m; ++k) c[k] = (k == j) ? 1.0 : 0.0;
+            return BC_OK;
+        }
+    }
+    double q[BC_MAX_K];
+    double sum = 0.0;
+    for (int j = 0; j < m; ++j) {
+        double prod = 1.0;
+        for (int k = 0; k < m; ++k)
+            if (k != j) prod *= (d[k] - d[j]);
+        q[j] = 1.0 / (prod * d[j]);
+        sum += q[j];
+    }
+    for (int j = 0; j < m; ++j) c[j] = q[j] / sum;
+    return BC_OK;
+}
+
+// Eqs. 8-12.  Node factors 1/2 at both ends of the window and 1 inside (Eq. 8); raw
+// weight with alternating sign, (-1)^j for j counted from 1 (Eq. 9); clip (Eq. 10);
+// signed decay power and normalisation (Eq. 11); blend towards x_{f=-1} (Eq. 12, read as
+// W = (1 - lambda) alpha + lambda e_1 so that the weights sum to one).
+bc_status solve_paper(const double *d, int m, const bc_params &p, double *c) {
+    const double delta = p.delta > 0.0 ? p.delta : delta_for_window(m);
+    double a[BC_MAX_K];
+    double sum = 0.0, mag = 0.0;
+    for (int j = 0; j < m; ++j) {
+        const double node_factor = (j == 0 || j == m - 1) ? 0.5 : 1.0;
+        const double alt = (j % 2 == 0) ? -1.0 : 1.0;  // (-1)^(j+1) for C index j
+        double u = node_factor * alt / d[j];
+        if (u > p.clip_C) u = p.clip_C;
+        if (u < -p.clip_C) u = -p.clip_C;
+        const double sg = u < 0.0 ? -1.0 : 1.0;
+        a[j] = sg * std::pow(std::fabs(u) + p.eta, delta);
+        sum += a[j];
+        mag += std::fabs(a[j]);
+    }
+    if (mag == 0.0 || !(std::fabs(sum) >= 1e-12 * mag))
+        return fail(BC_ERR_DEGENERATE_WEIGHTS, "Eq. 11 normaliser vanishes (sum %.3g of %.3g)",
+                    sum, mag);
+    for (int j = 0; j < m; ++j) c[j] = (1.0 - p.lambda) * (a[j] / sum);
+    c[0] += p.lambda;
+    return BC_OK;
+}
+
+bc_status solve_from_differences(const double *d, int m, const bc_params &p, double *c) {
+    for (int j = 0; j < m; ++j)
+        if (std::isnan(d[j])) return fail(BC_ERR_INVALID_ARG, "NaN timestep");
+    if (p.mode == BC_MODE_EXACT) return solve_exact(d, m, c);
+    return solve_paper(d, m, p, c);
+}
+
+// ------------------------------------------------------------------ Diff Key memo (Eq. 7)
+//
+// Key: the weight parameters and every difference t - s_j of the live window (the paper
+// prints H-1 differences; all H are needed to fix the weights, so all are keyed).
+struct Memo {
+    std::map<std::vector<double>, std::vector<double>> table;
+    int64_t hits = 0, misses = 0;
+    static constexpr size_t kCapacity = 4096;
+
+    bc_status lookup(const double *d, int m, const bc_params &p, double *c) {
+        std::vector<double> key = {static_cast<double>(p.mode), p.delta, p.lambda, p.clip_C,
+                                   p.eta, static_cast<double>(m)};
+        key.insert(key.end(), d, d + m);
+        auto it = table.find(key);
+        if (it != table.end()) {
+            ++hits;
+            std::memcpy(c, it->second.data(), sizeof(double) * m);
+            return BC_OK;
+        }
+        ++misses;
+        bc_status s = solve_from_differences(d, m, p, c);
+        if (s != BC_OK) return s;
+        if (table.size() >= kCapacity) table.clear();
+        table.emplace(std::move(key), std::vector<double>(c, c + m));
+        return BC_OK;
+    }
+};
+
+// ------------------------------------------------------------------ cache context (Eq. 6)
+
+constexpr uint64_t kAlign = 256;
+constexpr uint32_t kMagic = 0xBA7C0DE5u;
+
+int elem_bytes(bc_dtype d) { return d == BC_DTYPE_BF16 ? 2 : 4; }
+bool dtype_valid(int d) { return d == BC_DTYPE_F32 || d == BC_DTYPE_BF16; }
+uint64_t align_up(uint64_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
+
+bc_status layout(const int64_t *numels, int n_layers, int K, int dtype,
+                 std::vector<uint64_t> *offsets, uint64_t *slot_bytes) {
+    if (!numels || n_layers < 1) return fail(BC_ERR_INVALID_ARG, "need at least one layer");
+    if (K < 1 || K > BC_MAX_K) return fail(BC_ERR_INVALID_ARG, "K=%d outside 1..%d", K, BC_MAX_K);
+    if (!dtype_valid(dtype)) return fail(BC_ERR_INVALID_ARG, "unknown dtype %d", dtype);
+    const uint64_t eb = elem_bytes(static_cast<bc_dtype>(dtype));
+    const uint64_t kLimit = uint64_t(1) << 50;  // 1 PiB: far beyond any device
+    uint64_t off = 0;
+    if (offsets) offsets->clear();
+    for (int l = 0; l < n_layers; ++l) {
+        if (numels[l] < 0 || static_cast<uint64_t>(numels[l]) > kLimit / eb)
+            return fail(BC_ERR_INVALID_ARG, "layer %d numel %lld out of range", l,
+                        static_cast<long long>(numels[l]));
+        if (offsets) offsets->push_back(off);
+        off += align_up(static_cast<uint64_t>(numels[l]) * eb);
+        if (off > kLimit) return fail(BC_ERR_INVALID_ARG, "cache larger than 1 PiB");
+    }
+    *slot_bytes = off;
+    return BC_OK;
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) {
+            ok = false;
+            return;
+        }
+        if (prev != dev && cudaSetDevice(dev) != cudaSuccess) ok = false;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct bc_cache {
+    uint32_t magic = kMagic;
+    int n_layers = 0;
+    int K = 0;
+    bc_dtype dtype = BC_DTYPE_BF16;
+    bc_params params{};
+    int device = 0;
+    std::vector<int64_t> numel;
+    std::vector<uint64_t> offset;  // byte offset of each layer inside a slot
+    uint64_t slot_bytes = 0;
+    char *arena = nullptr;
+    uint64_t arena_bytes = 0;
+    int head = -1;                 // slot index of the newest node
+    int count = 0;                 // live nodes (<= K)
+    double node_t[BC_MAX_K] = {0, 0, 0, 0};
+    Memo memo;
+    bc_stats stats{};
+    std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
+
+    char *slot_base(int slot) const { return arena + static_cast<uint64_t>(slot) * slot_bytes; }
+    int slot_of_node(int j) const { return ((head - j) % K + K) % K; }  // j = 0 newest
+    bool overlaps_arena(uint64_t p, uint64_t bytes) const {
+        const uint64_t a0 = reinterpret_cast<uint64_t>(arena), a1 = a0 + arena_bytes;
+        return bytes != 0 && arena_bytes != 0 && p < a1 && a0 < p + bytes;
+    }
+};
+
+namespace {
+
+std::mutex g_registry_mu;
+std::unordered_set<bc_cache *> g_registry;
+
+bc_status check_handle(bc_handle h) {
+    if (!h) return fail(BC_ERR_BAD_HANDLE, "null handle");
+    std::lock_guard<std::mutex> lk(g_registry_mu);
+    if (!g_registry.count(h) || h->magic != kMagic)
+        return fail(BC_ERR_BAD_HANDLE, "handle is not a live cache");
+    return BC_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Weights for a forecast at t_new from the live window (through the memo).
+bc_status window_weights(bc_cache *h, double t_new, double *c, int *m) {
+    if (!std::isfinite(t_new)) return fail(BC_ERR_INVALID_ARG, "non-finite target timestep");
+    if (h->count == 0) return fail(BC_ERR_NOT_READY, "forecast before any push");
+    double d[BC_MAX_K];
+    for (int j = 0; j < h->count; ++j) d[j] = t_new - h->node_t[h->slot_of_node(j)];
+    *m = h->count;
+    return h->memo.lookup(d, h->count, h->params, c);
+}
+
+bc_status check_new_node(bc_cache *h, double t) {
+    if (!std::isfinite(t)) return fail(BC_ERR_INVALID_ARG, "non-finite timestep");
+    // Nodes that survive this push: all live ones, minus the oldest when the ring is full.
+    const int keep = h->count < h->K ? h->count : h->K - 1;
+    for (int j = 0; j < keep; ++j)
+        if (h->node_t[h->slot_of_node(j)] == t)
+            return fail(BC_ERR_DUPLICATE_NODE, "timestep %.17g already cached", t);
+    return BC_OK;
+}
+
+void rotate_in(bc_cache *h, double t) {
+    h->head = (h->head + 1) % h->K;
+    h->node_t[h->head] = t;
+    if (h->count < h->K) ++h->count;
+    ++h->stats.pushes;
+}
+
+bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_ptrs,
+                        bc_dtype out_dtype, int v_layer, void *x, bc_dtype x_dtype,
+                        void *stream) {
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!out_ptrs) return fail(BC_ERR_INVALID_ARG, "out_ptrs is NULL");
+    if (!dtype_valid(out_dtype)) return fail(BC_ERR_INVALID_ARG, "unknown output dtype");
+    const bool euler = v_layer >= 0;
+    if (euler) {
+        if (v_layer >= h->n_layers) return fail(BC_ERR_INVALID_ARG, "v_layer out of range");
+        if (!x) return fail(BC_ERR_INVALID_ARG, "x is NULL");
+        if (!dtype_valid(x_dtype)) return fail(BC_ERR_INVALID_ARG, "unknown x dtype");
+        if (!aligned16(x)) return fail(BC_ERR_ALIGNMENT, "x is not 16-byte aligned");
+        if (!std::isfinite(dt)) return fail(BC_ERR_INVALID_ARG, "non-finite dt");
+    }
+    double c[BC_MAX_K];
+    int m = 0;
+    s = window_weights(h, t_new, c, &m);
+    if (s != BC_OK) return s;
+
+    const uint64_t out_eb = elem_bytes(out_dtype);
+    const uint64_t x_bytes =
+        euler ? static_cast<uint64_t>(h->numel[v_layer]) * elem_bytes(x_dtype) : 0;
+    const uint64_t x0 = reinterpret_cast<uint64_t>(x);
+    if (euler && h->overlaps_arena(x0, x_bytes))
+        return fail(BC_ERR_INVALID_ARG, "x overlaps the cache arena");
+
+    auto &entries = h->scratch_entries;
+    entries.clear();
+    int euler_index = -1;
+    for (int l = 0; l < h->n_layers; ++l) {
+        void *o = out_ptrs[l];
+        if (!o && !(euler && l == v_layer)) continue;
+        const uint64_t ob = static_cast<uint64_t>(h->numel[l]) * out_eb;
+        if (o) {
+            if (!aligned16(o)) return fail(BC_ERR_ALIGNMENT, "output %d not 16-byte aligned", l);
+            const uint64_t p = reinterpret_cast<uint64_t>(o);
+            if (h->overlaps_arena(p, ob))
+                return fail(BC_ERR_INVALID_ARG, "output %d overlaps the cache arena", l);
+            if (euler && x_bytes && ob && p < x0 + x_bytes && x0 < p + ob)
+                return fail(BC_ERR_INVALID_ARG, "output %d aliases x", l);
+        }
+        if (euler && l == v_layer) euler_index = static_cast<int>(entries.size());
+        bc::LayerEntry e{};
+        e.src = h->offset[l];
+        e.dst = reinterpret_cast<uint64_t>(o);
+        e.numel = h->numel[l];
+        entries.push_back(e);
+    }
+
+    bc::LaunchPlan plan{};
+    for (int j = 0; j < BC_MAX_K; ++j) {
+        plan.slot[j] = j < m ? reinterpret_cast<uint64_t>(h->slot_base(h->slot_of_node(j))) : 0;
+        plan.w[j] = j < m ? static_cast<float>(c[j]) : 0.0f;
+    }
+    plan.K = m;
+    plan.in_dtype = h->dtype;
+    plan.out_dtype = out_dtype;
+    plan.dt = static_cast<float>(dt);
+    plan.euler_layer = euler_index;
+    plan.x_dtype = x_dtype;
+    plan.x = x0;
+    plan.layers = entries.data();
+    plan.n_layers = static_cast<int>(entries.size());
+
+    if (plan.n_layers > 0) {
+        DeviceGuard g(h->device);
+        if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+        const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches);
+        if (err != cudaSuccess) return cuda_fail(err, "forecast launch");
+    }
+    ++h->stats.forecasts;
+    h->stats.memo_hits = h->memo.hits;
+    h->stats.memo_misses = h->memo.misses;
+    return BC_OK;
+}
+
+}  // namespace
+
+// ======================================================================= C ABI
+extern "C" {
+
+int bc_version(void) { return 10000; }
+
+const char *bc_status_string(bc_status s) {
+    switch (s) {
+    case BC_OK: return "ok";
+    case BC_ERR_INVALID_ARG: return "invalid argument";
+    case BC_ERR_ALIGNMENT: return "device pointer not 16-byte aligned";
+    case BC_ERR_OOM: return "device allocation failed";
+    case BC_ERR_CUDA: return "CUDA runtime error";
+    case BC_ERR_NOT_READY: return "no feature pushed yet";
+    case BC_ERR_DUPLICATE_NODE: return "timestep already in the cache window";
+    case BC_ERR_DEGENERATE_WEIGHTS: return "weight normaliser vanishes";
+    case BC_ERR_BAD_HANDLE: return "bad handle";
+    }
+    return "unknown status";
+}
+
+const char *bc_last_error(void) { return t_last_error.c_str(); }
+
+void bc_params_default(bc_params *p) {
+    if (!p) return;
+    p->mode = BC_MODE_PAPER;
+    p->delta = 0.0;
+    p->lambda = 0.0;
+    p->clip_C = 10.0;
+    p->eta = 1e-12;
+}
+
+bc_status bc_solve(const double *nodes, int m, double t, const bc_params *p, double *c_out) {
+    t_last_error.clear();
+    try {
+        bc_params prm;
+        bc_params_default(&prm);
+        if (p) prm = *p;
+        if (!nodes || !c_out) return fail(BC_ERR_INVALID_ARG, "null pointer");
+        if (m < 1 || m > BC_MAX_K) return fail(BC_ERR_INVALID_ARG, "m=%d outside 1..%d", m, BC_MAX_K);
+        if (!params_valid(prm)) return fail(BC_ERR_INVALID_ARG, "invalid weight parameters");
+        if (!std::isfinite(t)) return fail(BC_ERR_INVALID_ARG, "non-finite target timestep");
+        double d[BC_MAX_K];
+        for (int j = 0; j < m; ++j) {
+            if (!std::isfinite(nodes[j])) return fail(BC_ERR_INVALID_ARG, "non-finite node");
+            d[j] = t - nodes[j];
+        }
+        return solve_from_differences(d, m, prm, c_out);
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
+                             int64_t *bytes) {
+    t_last_error.clear();
+    try {
+        if (!bytes) return fail(BC_ERR_INVALID_ARG, "bytes is NULL");
+        uint64_t slot = 0;
+        bc_status s = layout(numels, n_layers, K, dtype, nullptr, &slot);
+        if (s != BC_OK) return s;
+        *bytes = static_cast<int64_t>(slot * static_cast<uint64_t>(K));
+        return BC_OK;
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
+                          const bc_params *p, bc_handle *out) {
+    t_last_error.clear();
+    if (!out) return fail(BC_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    bc_cache *h = nullptr;
+    try {
+        bc_params prm;
+        bc_params_default(&prm);
+        if (p) prm = *p;
+        if (!params_valid(prm)) return fail(BC_ERR_INVALID_ARG, "invalid weight parameters");
+        std::vector<uint64_t> offs;
+        uint64_t slot = 0;
+        bc_status s = layout(numels, n_layers, K, dtype, &offs, &slot);
+        if (s != BC_OK) return s;
+        h = new bc_cache();
+        h->n_layers = n_layers;
+        h->K = K;
+        h->dtype = dtype;
+        h->params = prm;
+        h->numel.assign(numels, numels + n_layers);
+        h->offset = std::move(offs);
+        h->slot_bytes = slot;
+        h->arena_bytes = slot * static_cast<uint64_t>(K);
+        if (cudaGetDevice(&h->device) != cudaSuccess) {
+            delete h;
+            cudaGetLastError();
+            return fail(BC_ERR_CUDA, "no CUDA device");
+        }
+        if (h->arena_bytes > 0) {
+            void *mem = nullptr;
+            cudaError_t e = cudaMalloc(&mem, h->arena_bytes);
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                delete h;
+                if (e == cudaErrorMemoryAllocation)
+                    return fail(BC_ERR_OOM, "cannot allocate %llu bytes of cache",
+                                static_cast<unsigned long long>(slot * K));
+                return cuda_fail(e, "cudaMalloc");
+            }
+            h->arena = static_cast<char *>(mem);
+        }
+        {
+            std::lock_guard<std::mutex> lk(g_registry_mu);
+            g_registry.insert(h);
+        }
+        *out = h;
+        return BC_OK;
+    } catch (const std::bad_alloc &) {
+        delete h;
+        return fail(BC_ERR_OOM, "host allocation failed");
+    } catch (...) {
+        delete h;
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_cache_destroy(bc_handle h) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    {
+        std::lock_guard<std::mutex> lk(g_registry_mu);
+        g_registry.erase(h);
+    }
+    h->magic = 0;
+    bc_status rc = BC_OK;
+    if (h->arena) {
+        DeviceGuard g(h->device);
+        cudaError_t e = cudaDeviceSynchronize();
+        if (e == cudaSuccess) e = cudaFree(h->arena);
+        if (e != cudaSuccess) rc = cuda_fail(e, "cudaFree");
+    }
+    delete h;
+    return rc;
+}
+
+bc_status bc_cache_bytes(bc_handle h, int64_t *bytes) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!bytes) return fail(BC_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = static_cast<int64_t>(h->arena_bytes);
+    return BC_OK;
+}
+
+bc_status bc_cache_set_params(bc_handle h, const bc_params *p) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    bc_params prm;
+    bc_params_default(&prm);
+    if (p) prm = *p;
+    if (!params_valid(prm)) return fail(BC_ERR_INVALID_ARG, "invalid weight parameters");
+    h->params = prm;
+    h->memo.table.clear();
+    return BC_OK;
+}
+
+bc_status bc_cache_reset(bc_handle h) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    h->head = -1;
+    h->count = 0;
+    return BC_OK;
+}
+
+bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, void *stream) {
+    t_last_error.clear();
+    try {
+        bc_status s = check_handle(h);
+        if (s != BC_OK) return s;
+        if (!layer_ptrs) return fail(BC_ERR_INVALID_ARG, "layer_ptrs is NULL");
+        s = check_new_node(h, t);
+        if (s != BC_OK) return s;
+        const int next = (h->head + 1) % h->K;
+        const uint64_t eb = elem_bytes(h->dtype);
+        auto &entries = h->scratch_entries;
+        entries.clear();
+        for (int l = 0; l < h->n_layers; ++l) {
+            if (h->numel[l] == 0) continue;
+            const void *src = layer_ptrs[l];
+            if (!src) return fail(BC_ERR_INVALID_ARG, "layer %d source is NULL", l);
+            if (!aligned16(src)) return fail(BC_ERR_ALIGNMENT, "layer %d source not 16-byte aligned", l);
+            if (h->overlaps_arena(reinterpret_cast<uint64_t>(src), h->numel[l] * eb))
+                return fail(BC_ERR_INVALID_ARG, "layer %d source overlaps the cache arena", l);
+            bc::LayerEntry e{};
+            e.src = reinterpret_cast<uint64_t>(src);
+            e.dst = reinterpret_cast<uint64_t>(h->slot_base(next) + h->offset[l]);
+            e.numel = h->numel[l];
+            entries.push_back(e);
+        }
+        if (!entries.empty()) {
+            DeviceGuard g(h->device);
+            if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+            const int err = bc::launch_copy(entries.data(), static_cast<int>(entries.size()),
+                                            h->dtype, stream, &h->stats.kernel_launches);
+            if (err != cudaSuccess) return cuda_fail(err, "push copy launch");
+        }
+        rotate_in(h, t);
+        return BC_OK;
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_cache_next_slot_ptrs(bc_handle h, void **out_ptrs) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!out_ptrs) return fail(BC_ERR_INVALID_ARG, "out_ptrs is NULL");
+    const int next = (h->head + 1) % h->K;
+    for (int l = 0; l < h->n_layers; ++l) out_ptrs[l] = h->slot_base(next) + h->offset[l];
+    return BC_OK;
+}
+
+bc_status bc_cache_commit(bc_handle h, double t) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    s = check_new_node(h, t);
+    if (s != BC_OK) return s;
+    rotate_in(h, t);
+    return BC_OK;
+}
+
+bc_status bc_cache_nodes(bc_handle h, double *nodes_out, int *m_out) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!nodes_out || !m_out) return fail(BC_ERR_INVALID_ARG, "null pointer");
+    for (int j = 0; j < h->count; ++j) nodes_out[j] = h->node_t[h->slot_of_node(j)];
+    *m_out = h->count;
+    return BC_OK;
+}
+
+bc_status bc_cache_slot_ptrs(bc_handle h, int j, void **out_ptrs) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!out_ptrs) return fail(BC_ERR_INVALID_ARG, "out_ptrs is NULL");
+    if (j < 0 || j >= h->count) return fail(BC_ERR_INVALID_ARG, "node %d is not live", j);
+    char *base = h->slot_base(h->slot_of_node(j));
+    for (int l = 0; l < h->n_layers; ++l) out_ptrs[l] = base + h->offset[l];
+    return BC_OK;
+}
+
+bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out) {
+    t_last_error.clear();
+    try {
+        bc_status s = check_handle(h);
+        if (s != BC_OK) return s;
+        if (!c_out || !m_out) return fail(BC_ERR_INVALID_ARG, "null pointer");
+        s = window_weights(h, t_new, c_out, m_out);
+        h->stats.memo_hits = h->memo.hits;
+        h->stats.memo_misses = h->memo.misses;
+        return s;
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
+                      void *stream) {
+    t_last_error.clear();
+    try {
+        return forecast_impl(h, t_new, 0.0, out_ptrs, out_dtype, -1, nullptr, BC_DTYPE_F32,
+                             stream);
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_forecast_step(bc_handle h, double t_new, double dt, void *const *out_ptrs,
+                           bc_dtype out_dtype, int v_layer, void *x, bc_dtype x_dtype,
+                           void *stream) {
+    t_last_error.clear();
+    try {
+        if (v_layer < 0) return fail(BC_ERR_INVALID_ARG, "v_layer must name a cached layer");
+        return forecast_impl(h, t_new, dt, out_ptrs, out_dtype, v_layer, x, x_dtype, stream);
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_cache_stats(bc_handle h, bc_stats *out) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!out) return fail(BC_ERR_INVALID_ARG, "out is NULL");
+    h->stats.memo_hits = h->memo.hits;
+    h->stats.memo_misses = h->memo.misses;
+    *out = h->stats;
+    return BC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,264 @@
+"""GPU parity of the grouped forecast, the push copy and the fused Euler step.
+
+Every case builds seeded host features (numpy), pushes them through the C ABI, runs the
+CUDA path and compares each output element with the fp64 oracle on the same stored inputs:
+|gpu - oracle| <= 1e-5 * sum_j |W_j||F_j| for fp32 output, 2^-8 * sum_j |W_j||F_j| for bf16
+(and |x| + |dt| sum_j |W_j||V_j| for the Euler state).  Sizes span several tiles and
+ragged tails while keeping the oracle fast.
+"""
+from math import prod
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_28670_gb300 import barycache as bc
+from paper_2608_28670_gb300 import synth
+from tests.gpu_helpers import (as_f64, assert_close, device_view, empty_out, oracle_weights,
+                               stream, to_device, to_host)
+
+pytestmark = pytest.mark.gpu
+
+DT_NAME = {bc.DTYPE_F32: "f32", bc.DTYPE_BF16: "bf16"}
+# kTileVecs = 1024 vectors of 16 B: 8192 bf16 / 4096 f32 elements per tile.
+RAGGED = [1, 7, 8, 9, 4095, 4096, 4097, 8191, 8192, 8193, 3 * 8192 + 5, 100_003]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build_libraries()
+    torch.cuda.set_device(0)
+
+
+def run_case(numels, K, n_push, in_dt, out_dt, params, t_new, push_times, seed,
+             zero_copy=False, pad=64):
+    shapes = [(n,) for n in numels]
+    taus = list(push_times)
+    feats = synth.host_trajectories(shapes, taus, dtype=DT_NAME[in_dt], degree=2,
+                                    noise_std=1e-2, seed=seed)
+    h = bc.bc_cache_create(numels, K, in_dt, params)
+    try:
+        for i in range(n_push):
+            if zero_copy:
+                slots = bc.bc_cache_next_slot_ptrs(h, len(numels))
+                for l, n in enumerate(numels):
+                    if n:
+                        device_view(slots[l], n, in_dt).copy_(to_device(feats[i][l]))
+                bc.bc_cache_commit(h, push_times[i])
+            else:
+                dev = [to_device(f) for f in feats[i]]
+                bc.bc_cache_push(h, [d.data_ptr() for d in dev], push_times[i], stream())
+                torch.cuda.synchronize()   # `dev` may be freed after this
+        outs = [empty_out(n, out_dt, pad) for n in numels]
+        for o in outs:
+            o.fill_(0x5A5A if out_dt == bc.DTYPE_BF16 else 7.25)
+        ptrs = [o.data_ptr() + pad * o.element_size() for o in outs]
+        bc.bc_forecast(h, t_new, ptrs, out_dt, stream())
+        torch.cuda.synchronize()
+        m = min(n_push, K)
+        nodes = list(reversed(push_times[:n_push]))[:m]
+        got_nodes = bc.bc_cache_nodes(h)
+        assert got_nodes == nodes
+        W = oracle_weights(nodes, t_new, params.mode, lam=params.lambda_,
+                           delta=params.delta if params.delta > 0 else None,
+                           C=params.clip_C, eta=params.eta)
+        newest_first = [feats[i] for i in range(n_push - 1, n_push - 1 - m, -1)]
+        for l, n in enumerate(numels):
+            host = to_host(outs[l], out_dt)
+            canary = 0x5A5A if out_dt == bc.DTYPE_BF16 else np.float32(7.25)
+            assert np.all(host[:pad] == canary) and np.all(host[pad + n:] == canary), \
+                f"layer {l}: write outside the output"
+            if n == 0:
+                continue
+            ref, bound = oracle.combine([f[l] for f in newest_first], W)
+            assert_close(host[pad:pad + n], ref, bound, out_dt, f"layer {l} numel {n}")
+        return h
+    except Exception:
+        bc.bc_cache_destroy(h)
+        raise
+
+
+@pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+@pytest.mark.parametrize("out_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+@pytest.mark.parametrize("K", [1, 2, 3, 4])
+def test_ragged_layers_all_dtypes(in_dt, out_dt, K):
+    times = [0.9 - 0.05 * i for i in range(K)]
+    h = run_case(RAGGED, K, K, in_dt, out_dt, bc.make_params(), times[-1] - 0.05, times,
+                 seed=K * 10 + in_dt * 2 + out_dt)
+    bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("K", [2, 3, 4])
+@pytest.mark.parametrize("mode", [bc.MODE_EXACT, bc.MODE_PAPER])
+def test_partial_and_rotating_window(K, mode):
+    # Fewer pushes than K (m < K), exactly K, and K + 3 (the ring has wrapped).
+    for n_push in (1, K - 1, K, K + 3):
+        if n_push < 1:
+            continue
+        times = [980.0 - 20.0 * i for i in range(n_push)]
+        h = run_case([5000, 70_001], K, n_push, bc.DTYPE_BF16, bc.DTYPE_BF16,
+                     bc.make_params(mode=mode), times[-1] - 20.0, times, seed=n_push)
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("lam,delta,C", [(0.0, 0.0, 10.0), (0.5, 0.0, 10.0), (1.0, 0.0, 10.0),
+                                         (0.0, 0.7, 2.0), (0.2, 1.0, 10.0)])
+def test_weight_parameters_flow_time(lam, delta, C):
+    # Flow-matching time in [0, 1]: the clip of Eq. 10 is active at this spacing.
+    times = [1.0, 25 / 28, 22 / 28]
+    h = run_case([33_333, 8192], 3, 3, bc.DTYPE_BF16, bc.DTYPE_F32,
+                 bc.make_params(lam=lam, delta=delta, clip_C=C), 21 / 28, times, seed=5)
+    bc.bc_cache_destroy(h)
+
+
+def test_zero_copy_push():
+    times = [0.8, 0.7, 0.6, 0.5, 0.4]
+    h = run_case([12_345, 1, 65_536], 3, 5, bc.DTYPE_BF16, bc.DTYPE_BF16, bc.make_params(),
+                 0.35, times, seed=11, zero_copy=True)
+    bc.bc_cache_destroy(h)
+
+
+def test_exact_mode_node_hit_returns_the_node():
+    times = [0.8, 0.7, 0.6]
+    h = run_case([10_000], 3, 3, bc.DTYPE_F32, bc.DTYPE_F32, bc.make_params(mode=bc.MODE_EXACT),
+                 0.7, times, seed=3)
+    try:
+        out = torch.empty(10_000, dtype=torch.float32, device="cuda")
+        bc.bc_forecast(h, 0.7, [out.data_ptr()], bc.DTYPE_F32, stream())
+        slot = device_view(bc.bc_cache_slot_ptrs(h, 1, 1)[0], 10_000, bc.DTYPE_F32)
+        torch.cuda.synchronize()
+        assert torch.equal(out, slot)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_push_copy_is_byte_exact():
+    # Includes NaN payloads and -0.0: the push must move bytes, not values.
+    n = 3 * 8192 + 3
+    rng = np.random.default_rng(1)
+    bits = rng.integers(0, 2 ** 16, n, dtype=np.uint16)
+    bits[:4] = [0x7FC1, 0xFFFF, 0x8000, 0x7F80]
+    h = bc.bc_cache_create([n, n + 1], 2, bc.DTYPE_BF16)
+    try:
+        src = [to_device(bits), to_device(np.concatenate([bits, bits[:1]]))]
+        bc.bc_cache_push(h, [s.data_ptr() for s in src], 0.5, stream())
+        torch.cuda.synchronize()
+        slots = bc.bc_cache_slot_ptrs(h, 0, 2)
+        for l, s in enumerate(src):
+            got = device_view(slots[l], s.numel(), bc.DTYPE_BF16)
+            assert torch.equal(got, s)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_null_outputs_skip_layers_and_window_forecast():
+    numels = [8192 * 3, 1000, 77_777, 64]
+    times = [0.9, 0.8, 0.7]
+    h = run_case(numels, 3, 3, bc.DTYPE_BF16, bc.DTYPE_BF16, bc.make_params(), 0.65, times, seed=8)
+    try:
+        outs = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        for o in outs:
+            o.fill_(123)
+        ptrs = [outs[0].data_ptr(), None, outs[2].data_ptr(), None]
+        before = bc.bc_cache_stats(h)["kernel_launches"]
+        bc.bc_forecast(h, 0.65, ptrs, bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["kernel_launches"] == before + 1
+        assert torch.all(outs[1] == 123) and torch.all(outs[3] == 123)
+        assert not torch.all(outs[0] == 123)
+        # no output at all: nothing is launched
+        bc.bc_forecast(h, 0.65, [None] * 4, bc.DTYPE_BF16, stream())
+        assert bc.bc_cache_stats(h)["kernel_launches"] == before + 1
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_many_layers_use_several_launches():
+    numels = [(i * 37) % 301 + 1 for i in range(300)]   # 300 tiny ragged layers
+    times = [0.9, 0.85]
+    h = run_case(numels, 2, 2, bc.DTYPE_F32, bc.DTYPE_BF16, bc.make_params(), 0.8, times, seed=9)
+    try:
+        s0 = bc.bc_cache_stats(h)["kernel_launches"]
+        outs = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        bc.bc_forecast(h, 0.8, [o.data_ptr() for o in outs], bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["kernel_launches"] - s0 == 2   # 240 + 60 layers
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("x_dt", [bc.DTYPE_F32, bc.DTYPE_BF16])
+@pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+@pytest.mark.parametrize("store_v", [False, True])
+def test_fused_euler_step(x_dt, in_dt, store_v):
+    numels = [8192 * 2 + 3, 262_144 + 5]   # a block output and a ragged "velocity"
+    times = [1.0, 25 / 28, 22 / 28]
+    t_new, dt = 21 / 28, -1 / 28
+    feats = synth.host_trajectories([(n,) for n in numels], times, dtype=DT_NAME[in_dt], seed=21)
+    x0 = synth.host_trajectories([(numels[1],)], [0.0], dtype=DT_NAME[x_dt], degree=0,
+                                 noise_std=0.0, seed=22)[0][0]
+    h = bc.bc_cache_create(numels, 3, in_dt)
+    try:
+        for t, per in zip(times, feats):
+            dev = [to_device(f) for f in per]
+            bc.bc_cache_push(h, [d.data_ptr() for d in dev], t, stream())
+            torch.cuda.synchronize()
+        out0 = empty_out(numels[0], bc.DTYPE_F32)
+        vout = empty_out(numels[1], bc.DTYPE_F32) if store_v else None
+        x = to_device(x0)
+        s0 = bc.bc_cache_stats(h)["kernel_launches"]
+        bc.bc_forecast_step(h, t_new, dt, [out0.data_ptr(), vout.data_ptr() if store_v else None],
+                            bc.DTYPE_F32, 1, x.data_ptr(), x_dt, stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["kernel_launches"] - s0 == 1
+        W = oracle.paper_weights(list(reversed(times)), t_new)
+        nf = feats[::-1]
+        ref, bound = oracle.combine([f[0] for f in nf], W)
+        assert_close(to_host(out0, bc.DTYPE_F32), ref, bound, bc.DTYPE_F32, "block")
+        x_ref, v_ref, xb = oracle.euler([f[1] for f in nf], W, x0, dt)
+        assert_close(to_host(x, x_dt), x_ref, xb, x_dt, "x")
+        if store_v:
+            _, vb = oracle.combine([f[1] for f in nf], W)
+            assert_close(to_host(vout, bc.DTYPE_F32), v_ref, vb, bc.DTYPE_F32, "v_hat")
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_memo_reuses_weights_across_the_schedule():
+    # Same differences t - s_j at a later point of an equal-spaced schedule: a memo hit.
+    h = bc.bc_cache_create([1024], 2, bc.DTYPE_BF16)
+    try:
+        z = torch.zeros(1024, dtype=torch.int16, device="cuda")
+        bc.bc_cache_push(h, [z.data_ptr()], 0.9, stream())
+        bc.bc_cache_push(h, [z.data_ptr()], 0.84, stream())
+        c1 = bc.bc_coefficients(h, 0.82)
+        bc.bc_cache_push(h, [z.data_ptr()], 0.78, stream())
+        c2 = bc.bc_coefficients(h, 0.76)
+        torch.cuda.synchronize()
+        st = bc.bc_cache_stats(h)
+        assert st["memo_misses"] >= 1
+        # the differences are (0.02, 0.08) up to rounding of the time grid
+        np.testing.assert_allclose(c1, c2, rtol=1e-9)
+        c3 = bc.bc_coefficients(h, 0.76)
+        assert c3 == c2 and bc.bc_cache_stats(h)["memo_hits"] >= st["memo_hits"] + 1
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_empty_layers_and_footprint():
+    numels = [0, 5, 0]
+    h = bc.bc_cache_create(numels, 2, bc.DTYPE_F32)
+    try:
+        assert bc.bc_cache_bytes(h) == bc.bc_cache_bytes_for(numels, 2, bc.DTYPE_F32) == 512
+        x = torch.arange(5, dtype=torch.float32, device="cuda")
+        bc.bc_cache_push(h, [0, x.data_ptr(), 0], 1.0, stream())
+        bc.bc_cache_push(h, [0, (x * 2).data_ptr(), 0], 0.5, stream())
+        out = torch.empty(5, dtype=torch.float32, device="cuda")
+        bc.bc_forecast(h, 0.0, [None, out.data_ptr(), None], bc.DTYPE_F32, stream())
+        torch.cuda.synchronize()
+        # x(t) = (2 - 2t) * x_base is linear in t: the H = 2 forecast at t = 0 is 2 * x_base
+        np.testing.assert_allclose(out.cpu().numpy(), 3.0 * np.arange(5), rtol=1e-6)
+    finally:
+        bc.bc_cache_destroy(h)

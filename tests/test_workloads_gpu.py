@@ -1,0 +1,130 @@
+"""Full-size parity of the five workloads, in the launch configuration the benchmark times.
+
+The history slots are written in place by the seeded device generator (never by the
+forecast path); the forecast runs through the C ABI exactly as in ``bench.py``; then, per
+layer, a sample of element indices (first, last, the ragged end of every tile boundary
+region and random positions) is gathered from the stored inputs and the outputs and
+checked against the fp64 oracle element by element.  The DiT-XL/2 256 px case is small
+enough to check every element.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_28670_gb300 import barycache as bc
+from paper_2608_28670_gb300.configs import WORKLOADS, T2V_HBM_BUDGET
+from paper_2608_28670_gb300.runner import WorkloadRun
+from tests.gpu_helpers import as_f64, assert_close, device_view, oracle_weights, stream
+
+pytestmark = pytest.mark.gpu
+SAMPLES = 4096
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build_libraries()
+    torch.cuda.set_device(0)
+
+
+def sample_indices(n: int, rng) -> torch.Tensor:
+    fixed = [0, 1, n // 2, n - 2, n - 1] + [min(n - 1, k * 8192 + d) for k in (1, 2, 3)
+                                               for d in (-1, 0, 1)]
+    idx = np.unique(np.concatenate([np.array(fixed), rng.integers(0, n, SAMPLES)]))
+    return torch.from_numpy(idx[(idx >= 0) & (idx < n)]).cuda()
+
+
+def gather(ptr: int, n: int, dtype: int, idx: torch.Tensor) -> np.ndarray:
+    v = device_view(ptr, n, dtype)[idx]
+    a = v.cpu().numpy()
+    return a.view(np.uint16) if dtype == bc.DTYPE_BF16 else a
+
+
+def check_run(run: WorkloadRun, rng, calls=None):
+    w, h = run.w, run.h
+    p = run.problem
+    W = oracle_weights(list(p.nodes), p.t, bc.MODE_PAPER)
+    assert bc.bc_cache_nodes(h) == list(p.nodes)
+    m = len(p.nodes)
+    slot_ptrs = [bc.bc_cache_slot_ptrs(h, j, len(run.numels)) for j in range(m)]
+    calls = range(run.calls) if calls is None else calls
+    if run.euler:
+        x_before = run.x.clone()
+    out_dt = bc.DTYPE_BF16 if run.out_dtype == bc.DTYPE_BF16 else bc.DTYPE_F32
+    for c in calls:
+        run.forecast_call(c)
+        torch.cuda.synchronize()
+        for i in range(run.window):
+            l = c * run.window + i
+            if l >= run.n_feat:
+                break
+            n = run.numels[l]
+            idx = sample_indices(n, rng)
+            F = [gather(slot_ptrs[j][l], n, w.dtype, idx) for j in range(m)]
+            ref, bound = oracle.combine(F, W)
+            outv = run.outs[i].view(torch.int16) if out_dt == bc.DTYPE_BF16 else run.outs[i]
+            got = outv[idx].cpu().numpy()
+            got = got.view(np.uint16) if out_dt == bc.DTYPE_BF16 else got
+            assert_close(got, ref, bound, out_dt, f"{w.name} layer {l}")
+        if run.euler and c == 0:
+            nv = run.numels[-1]
+            idx = torch.arange(nv, device="cuda")
+            V = [gather(slot_ptrs[j][-1], nv, w.dtype, idx) for j in range(m)]
+            x_ref, _, xb = oracle.euler(V, W, x_before.cpu().numpy(), p.dt)
+            assert_close(run.x.cpu().numpy(), x_ref, xb, bc.DTYPE_F32, f"{w.name} Euler x")
+
+
+def test_c2i_256_every_element():
+    w = WORKLOADS["c2i-256"]
+    run = WorkloadRun(w, stream=stream())
+    try:
+        run.forecast()
+        torch.cuda.synchronize()
+        p = run.problem
+        assert p.nodes == (940.0, 960.0, 980.0) and p.t == 920.0
+        W = oracle_weights(list(p.nodes), p.t, bc.MODE_PAPER)
+        n = w.layer_numel
+        F = [device_view(bc.bc_cache_slot_ptrs(run.h, j, 1)[0], n, w.dtype).cpu().numpy()
+             for j in range(3)]
+        ref, bound = oracle.combine(F, W)
+        assert_close(run.outs[0].cpu().numpy(), ref, bound, bc.DTYPE_F32, "c2i-256")
+        # Exact mode recovers the quadratic trajectory: W = (3, -3, 1) exactly.
+        bc.bc_cache_set_params(run.h, bc.make_params(mode=bc.MODE_EXACT))
+        assert bc.bc_coefficients(run.h, 920.0) == [3.0, -3.0, 1.0]
+    finally:
+        run.close()
+
+
+@pytest.mark.parametrize("name", ["c2i-512", "t2i-1024", "mmdit-t2i"])
+def test_image_workloads_sampled(name):
+    torch.cuda.empty_cache()
+    run = WorkloadRun(WORKLOADS[name], stream=stream())
+    try:
+        assert run.calls == 1
+        check_run(run, np.random.default_rng(len(name)))
+        st = run.stats()
+        assert st["kernel_launches"] == 1 and st["forecasts"] == 1
+    finally:
+        run.close()
+        torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("K", [2, 3, 4])
+def test_t2v_sampled_within_budget(K):
+    torch.cuda.empty_cache()
+    free, _ = torch.cuda.mem_get_info()
+    w = WORKLOADS["t2v"]
+    if free < w.cache_bytes(K) + 8 * 10**9:
+        pytest.skip(f"needs {w.cache_bytes(K) / 1e9:.0f} GB free, have {free / 1e9:.0f} GB")
+    run = WorkloadRun(w, K=K, budget_bytes=T2V_HBM_BUDGET, stream=stream())
+    try:
+        total = bc.bc_cache_bytes(run.h) + run.window * w.layer_numel * 2
+        assert total <= T2V_HBM_BUDGET
+        if K <= 3:
+            assert run.calls == 1
+        calls = sorted({0, run.calls // 2, run.calls - 1})
+        check_run(run, np.random.default_rng(K), calls=calls)
+    finally:
+        run.close()
+        torch.cuda.empty_cache()
