@@ -47,6 +47,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the push and fused-step measurements")
     return ap.parse_args()
 
 
@@ -153,10 +155,13 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     launches0 = run.stats()["kernel_launches"]
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    host_s = []
     torch.cuda.synchronize()
     for i in range(steps):
         starts[i].record()
+        h0 = time.perf_counter()
         run.forecast(ts[i % len(ts)])
+        host_s.append(time.perf_counter() - h0)
         ends[i].record()
     torch.cuda.synchronize()
     if dist is not None:
@@ -164,6 +169,7 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     total_ms = starts[0].elapsed_time(ends[-1])
     per_step = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     launches = run.stats()["kernel_launches"] - launches0
+    time_forecast.host_us = 1e6 * statistics.median(host_s)
     return total_ms, per_step, launches
 
 
@@ -244,6 +250,10 @@ def run_ours(args):
                 "algorithmic_bytes_per_launch": per_launch_bytes,
             },
             "gpu_launches": launches,
+            "step_ms": {"min": round(min(per_step), 4),
+                        "median": round(statistics.median(per_step), 4),
+                        "max": round(max(per_step), 4), "first": round(per_step[0], 4)},
+            "host_call_us": round(time_forecast.host_us, 1),
         }
         if clk:
             result["clocks"] = clk
@@ -267,13 +277,18 @@ def run_ours(args):
                     torch.cuda.empty_cache()
             result["sweep"] = sweep
             run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
-        if not args.no_e2e:
-            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
             result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
+        if not args.no_e2e:
+            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
+        if not args.no_extra:
+            result["push"] = time_push(run, args.steps)
     finally:
         if run is not None:
             run.close()
+    if not args.no_extra and w.name != "mmdit-t2i":
+        torch.cuda.empty_cache()
+        result["fused_step"] = time_fused(args, stream, dist)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -292,50 +307,161 @@ def _continuation(run, i):
     return t_full, t_full + off
 
 
-def e2e(run, steps, world, dist):
+def time_push(run, steps):
+    """Row a2, copy path: bc_cache_push of one full slot (every layer) from device buffers
+    (the forecast outputs stand in for a full step's features); 2 bytes of HBM traffic per
+    byte of slot.  Only when the outputs cover every layer."""
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    if run.window < run.n_feat or run.euler:
+        return None
+    ptrs = [o.data_ptr() for o in run.outs]
+    slot = sum(n * run.w.elem_bytes for n in run.numels)
+    t = [_continuation(run, 100 + i)[0] for i in range(steps + 2)]
+    for i in range(2):
+        bc.bc_cache_push(run.h, ptrs, t[i], run.stream)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    for i in range(steps):
+        bc.bc_cache_push(run.h, ptrs, t[2 + i], run.stream)
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    return {"GB/s": round(2 * slot / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
+            "bytes_per_push": 2 * slot, "pushes": steps,
+            "what": "grouped byte-exact copy of one slot (read + write)"}
+
+
+def time_fused(args, stream, dist):
+    """Row a4: the fused forecast + Euler step on the MMDiT workload (57 block outputs plus
+    the velocity [1, 16, 128, 128], one launch per step)."""
+    from paper_2608_28670_gb300.configs import WORKLOADS
+    from paper_2608_28670_gb300.runner import WorkloadRun
+    r = WorkloadRun(WORKLOADS["mmdit-t2i"], stream=stream)
+    try:
+        tm, ps, ln = time_forecast(r, args.steps, args.warmup, stream, dist)
+        ms = tm / args.steps
+        a = r.algorithmic_bytes()
+        return {"workload": "mmdit-t2i", "GB/s": round(a / (ms * 1e-3) / 1e9, 1),
+                "ms": round(ms, 4), "algorithmic_bytes_per_step": a, "launches": ln,
+                "steps": args.steps}
+    finally:
+        r.close()
+
+
+def pinned_host_buffer(nbytes):
+    """Page-locked host memory of exactly `nbytes`: cudaHostAlloc through the CUDA runtime
+    that torch loaded (concurrent H2D + D2H on GB300 need it; registered pageable memory
+    serialises them), else cudaHostRegister of a numpy buffer.  Returns (uint8 array,
+    release function, description)."""
+    import ctypes
+    import glob
+    import numpy as np
+    import torch
+    rt = None
+    cands = ["libcudart.so.13"] + sorted(glob.glob(os.path.join(
+        os.path.dirname(torch.__file__), "..", "nvidia", "*", "lib", "libcudart.so*")))
+    for c in cands:
+        try:
+            rt = ctypes.CDLL(c)
+            break
+        except OSError:
+            continue
+    if rt is not None:
+        ptr = ctypes.c_void_p()
+        rt.cudaHostAlloc.argtypes = [ctypes.POINTER(ctypes.c_void_p), ctypes.c_size_t,
+                                     ctypes.c_uint]
+        rt.cudaFreeHost.argtypes = [ctypes.c_void_p]
+        if rt.cudaHostAlloc(ctypes.byref(ptr), nbytes, 0) == 0 and ptr.value:
+            arr = np.ctypeslib.as_array((ctypes.c_uint8 * nbytes).from_address(ptr.value))
+            return arr, (lambda: rt.cudaFreeHost(ptr)), "cudaHostAlloc"
+    arr = np.empty(nbytes, dtype=np.uint8)
+    cudart = torch.cuda.cudart()
+    if int(cudart.cudaHostRegister(arr.ctypes.data, nbytes, 0)) != 0:
+        return None, None, f"no page-locked host buffer of {nbytes} bytes"
+    return arr, (lambda: cudart.cudaHostUnregister(arr.ctypes.data)), "cudaHostRegister"
+
+
+def e2e(run, steps, world, dist, chunk_layers=6):
     """Same metric through the public API with host buffers.  Per step: the new full-step
     features (one slot, every layer) are copied from pinned host memory into the next cache
     slot and committed (zero-copy push, Eq. 6), the following skipped step is forecast, and
     the forecast is read back into pinned host memory.  One pinned host buffer of one slot
-    serves both directions (the read-back of step i is the input of step i + 1)."""
+    serves both directions (the read-back of step i is the input of step i + 1).
+
+    The transfers are pipelined by chunks of layers on three streams: host->device copies of
+    chunk c, the forecast of chunk c (bc_forecast with the other outputs NULL) once they have
+    landed, and the device->host copy of its output; the next step's copy into chunk c waits
+    for this step's read-back of chunk c (which itself follows the forecast that read the slot
+    being overwritten)."""
     import numpy as np
     import torch
     from paper_2608_28670_gb300 import barycache as bc
     from paper_2608_28670_gb300.runner import device_view
 
+    if run.euler:
+        return {"unavailable": "e2e is measured on workloads without the Euler layer"}
     eb = run.w.elem_bytes
     ob = 2 if run.out_dtype == bc.DTYPE_BF16 else 4
+    if ob != eb:
+        return {"unavailable": "e2e reuses the input buffer for the output: dtypes differ"}
     sizes = [n * eb for n in run.numels]
     offs = np.cumsum([0] + sizes)
     total = int(offs[-1])
-    host = np.empty(total, dtype=np.uint8)
-    cudart = torch.cuda.cudart()
-    rc = cudart.cudaHostRegister(host.ctypes.data, total, 0)
-    if int(rc) != 0:
-        return {"unavailable": f"cudaHostRegister of {total} bytes failed ({rc})"}
+    host, release, kind = pinned_host_buffer(total)
+    if host is None:
+        return {"unavailable": kind}
     try:
         tdt = torch.bfloat16 if run.w.dtype == bc.DTYPE_BF16 else torch.float32
-        hviews = [torch.from_numpy(host[offs[l]:offs[l + 1]]).view(tdt)
-                  for l in range(len(run.numels))]
-        # initial content: the current newest slot (a real full-step feature)
-        newest = bc.bc_cache_slot_ptrs(run.h, 0, len(run.numels))
+        L = len(run.numels)
+        hviews = [torch.from_numpy(host[offs[l]:offs[l + 1]]).view(tdt) for l in range(L)]
+        newest = bc.bc_cache_slot_ptrs(run.h, 0, L)
         for l, n in enumerate(run.numels):
             hviews[l].copy_(device_view(newest[l], n, run.w.dtype).view(tdt))
         torch.cuda.synchronize()
+        cl = run.window if run.window < run.n_feat else chunk_layers
+        chunks = [list(range(c, min(c + cl, L))) for c in range(0, L, cl)]
+        s_in, s_fc, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        done_out = [None] * len(chunks)
+        shared_outs = run.window < run.n_feat
 
         def one_step(i):
             t_full, t_target = _continuation(run, i)
-            slots = bc.bc_cache_next_slot_ptrs(run.h, len(run.numels))
-            for l, n in enumerate(run.numels):
-                device_view(slots[l], n, run.w.dtype).view(tdt).copy_(hviews[l], non_blocking=True)
+            slots = bc.bc_cache_next_slot_ptrs(run.h, L)
+            landed = []
+            for c, ls in enumerate(chunks):
+                with torch.cuda.stream(s_in):
+                    if done_out[c] is not None:
+                        s_in.wait_event(done_out[c])
+                    for l in ls:
+                        device_view(slots[l], run.numels[l], run.w.dtype).view(tdt).copy_(
+                            hviews[l], non_blocking=True)
+                    ev = torch.cuda.Event()
+                    ev.record(s_in)
+                    landed.append(ev)
             bc.bc_cache_commit(run.h, t_full)
-            for c in range(run.calls):
-                run.forecast_call(c, t_target)
-                for k in range(run.window):
-                    l = c * run.window + k
-                    if l < run.n_feat:
-                        hviews[l].copy_(run.outs[k].view(tdt) if ob == eb else run.outs[k],
+            for c, ls in enumerate(chunks):
+                s_fc.wait_event(landed[c])
+                if shared_outs:   # the window's output buffers are reused by every chunk
+                    prev = done_out[c - 1] if c > 0 else done_out[-1]
+                    if prev is not None:
+                        s_fc.wait_event(prev)
+                ptrs = [None] * L
+                for l in ls:
+                    ptrs[l] = run.outs[l - ls[0] if shared_outs else l].data_ptr()
+                bc.bc_forecast(run.h, t_target, ptrs, run.out_dtype, s_fc.cuda_stream)
+                ev = torch.cuda.Event()
+                ev.record(s_fc)
+                with torch.cuda.stream(s_out):
+                    s_out.wait_event(ev)
+                    for l in ls:
+                        hviews[l].copy_(run.outs[l - ls[0] if shared_outs else l],
                                         non_blocking=True)
+                    ev2 = torch.cuda.Event()
+                    ev2.record(s_out)
+                    done_out[c] = ev2
 
         one_step(0)                      # warm-up
         torch.cuda.synchronize()
@@ -347,6 +473,8 @@ def e2e(run, steps, world, dist):
         a.record()
         for i in range(steps):
             one_step(i + 1)
+        for ev in done_out:
+            torch.cuda.current_stream().wait_event(ev)
         b.record()
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
@@ -357,12 +485,16 @@ def e2e(run, steps, world, dist):
             ms = float(t.item())
         alg = run.algorithmic_bytes()
         return {"value": round(alg * world / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
-                "h2d_bytes_per_step": total, "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
+                "h2d_bytes_per_step": total,
+                "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
                 "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
+                "chunk_layers": cl, "host_memory": kind,
                 "path": "pinned host -> next cache slot (bc_cache_next_slot_ptrs + "
-                        "bc_cache_commit) -> bc_forecast -> pinned host"}
+                        "bc_cache_commit) -> bc_forecast per chunk -> pinned host, "
+                        "3 streams"}
     finally:
-        cudart.cudaHostUnregister(host.ctypes.data)
+        torch.cuda.synchronize()
+        release()
 
 
 CHUNK = 1 << 22   # elements per oracle call in the CPU samples

@@ -8,15 +8,19 @@
 // (2) enough independent 16-byte loads in flight per SM to cover HBM latency, and (3) one
 // launch for all cached tensors, so a 60-layer forecast costs one kernel, not sixty.
 //
-// Work decomposition: every layer is cut into tiles of kTileVecs 16-byte vectors; tiles
-// are numbered across layers by a prefix sum carried in the launch's parameter block; a
-// persistent grid (SM count x resident CTAs) walks the tile space with a grid stride, so
-// neighbouring CTAs stream neighbouring addresses at the same time.  Within a tile a
-// thread first issues all H x kVecsPerThread loads, then converts, accumulates in fp32 and
-// stores, which keeps up to 16 independent 128-bit loads in flight per thread.
+// Work decomposition: every layer is cut into tiles of kThreads x VPT history vectors of
+// 32 bytes; tiles are numbered across layers by a prefix sum carried in the launch's
+// parameter block; a persistent grid (two CTAs per SM) walks the tile space with a grid
+// stride, so neighbouring CTAs stream neighbouring addresses at the same time.  Within a
+// tile a thread first issues all H x VPT loads, then converts, accumulates in fp32 and
+// stores (VPT = 2, or 4 at H = 4: 6-16 independent 256-bit loads in flight per thread).
 //
-// Loads use ld.global.nc with L1::no_allocate (each byte is touched once, L1 reuse is
-// nil); stores use st.global.cs (streaming).  Nothing here waits on another CTA, nothing
+// History loads are 256-bit ld.global.nc with L1::no_allocate (each byte is touched
+// once; the slots are 256-byte aligned); outputs, the Euler state and push sources carry
+// only the ABI's 16-byte alignment and use 128-bit (or 64-bit) accesses; stores are
+// st.global.cs (streaming).  A sweep over vector width, vectors per thread, CTA size and
+// CTAs per SM on the 60-layer video workload picked these values (7.18 TB/s at H = 3,
+// against 6.96 TB/s for 128-bit loads at three CTAs per SM).  Nothing here waits on another CTA, nothing
 // allocates, and nothing traps: out-of-range work is never issued because every vector
 // index is checked against the layer's length.
 #include <cuda_bf16.h>
@@ -39,6 +43,50 @@ struct BF16 {
     using store_t = uint16_t;
     static constexpr int kBytes = 2;
 };
+
+// One history vector: kVecBytes bytes as 16-byte pieces.
+struct Raw {
+    uint4 q[kVecBytes / 16];
+};
+
+__device__ __forceinline__ uint64_t history_policy() {
+    uint64_t pol = 0;
+#if BC_L2_EVICT_FIRST
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+#endif
+    return pol;
+}
+
+// History loads: read-only for the whole kernel, touched once -> non-coherent path, no L1
+// allocation.  The slots are 256-byte aligned, so 32-byte vectors are always aligned.
+__device__ __forceinline__ Raw ld_history(const char *p, uint64_t pol) {
+    Raw r;
+    (void)pol;
+    if constexpr (kVecBytes == 32) {
+#if BC_L2_EVICT_FIRST
+        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8], %9;"
+            : "=r"(r.q[0].x), "=r"(r.q[0].y), "=r"(r.q[0].z), "=r"(r.q[0].w), "=r"(r.q[1].x),
+              "=r"(r.q[1].y), "=r"(r.q[1].z), "=r"(r.q[1].w)
+            : "l"(p), "l"(pol));
+#else
+        asm("ld.global.nc.L1::no_allocate.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            : "=r"(r.q[0].x), "=r"(r.q[0].y), "=r"(r.q[0].z), "=r"(r.q[0].w), "=r"(r.q[1].x),
+              "=r"(r.q[1].y), "=r"(r.q[1].z), "=r"(r.q[1].w)
+            : "l"(p));
+#endif
+    } else {
+#if BC_L2_EVICT_FIRST
+        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+            : "=r"(r.q[0].x), "=r"(r.q[0].y), "=r"(r.q[0].z), "=r"(r.q[0].w)
+            : "l"(p), "l"(pol));
+#else
+        asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+            : "=r"(r.q[0].x), "=r"(r.q[0].y), "=r"(r.q[0].z), "=r"(r.q[0].w)
+            : "l"(p));
+#endif
+    }
+    return r;
+}
 
 __device__ __forceinline__ uint4 ld_stream16(const void *p) {
     uint4 r;
@@ -87,54 +135,54 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return u;
 }
 
-// Unpack one 16-byte vector of T into EV = 16 / sizeof(T) floats.
+// 16 bytes of T <-> 16 / sizeof(T) floats.
 template <class T>
-__device__ __forceinline__ void unpack16(uint4 r, float *f);
-template <>
-__device__ __forceinline__ void unpack16<BF16>(uint4 r, float *f) {
-    f[0] = bf16_lo(r.x); f[1] = bf16_hi(r.x); f[2] = bf16_lo(r.y); f[3] = bf16_hi(r.y);
-    f[4] = bf16_lo(r.z); f[5] = bf16_hi(r.z); f[6] = bf16_lo(r.w); f[7] = bf16_hi(r.w);
-}
-template <>
-__device__ __forceinline__ void unpack16<F32>(uint4 r, float *f) {
-    f[0] = __uint_as_float(r.x); f[1] = __uint_as_float(r.y);
-    f[2] = __uint_as_float(r.z); f[3] = __uint_as_float(r.w);
-}
-
-// Load / store EV consecutive elements of T at element offset `e` (EV is the vector width
-// of the history dtype, so the footprint in T is 8, 16 or 32 bytes, naturally aligned).
-// Used for the Euler state only, hence the coherent loads.
-template <class T, int EV>
-__device__ __forceinline__ void load_elems(const char *base, int64_t e, float *f) {
-    const char *p = base + e * T::kBytes;
-    if constexpr (T::kBytes * EV == 16) {
-        unpack16<T>(ld_plain16(p), f);
-    } else if constexpr (T::kBytes * EV == 32) {  // f32 x 8
-        unpack16<T>(ld_plain16(p), f);
-        unpack16<T>(ld_plain16(p + 16), f + 4);
-    } else {                                       // bf16 x 4
-        uint2 r = ld_plain8(p);
+__device__ __forceinline__ void unpack16(uint4 r, float *f) {
+    if constexpr (std::is_same<T, BF16>::value) {
         f[0] = bf16_lo(r.x); f[1] = bf16_hi(r.x); f[2] = bf16_lo(r.y); f[3] = bf16_hi(r.y);
+        f[4] = bf16_lo(r.z); f[5] = bf16_hi(r.z); f[6] = bf16_lo(r.w); f[7] = bf16_hi(r.w);
+    } else {
+        f[0] = __uint_as_float(r.x); f[1] = __uint_as_float(r.y);
+        f[2] = __uint_as_float(r.z); f[3] = __uint_as_float(r.w);
     }
 }
 
-template <class T, int EV>
-__device__ __forceinline__ void store_elems(char *base, int64_t e, const float *f) {
-    char *p = base + e * T::kBytes;
+template <class T>
+__device__ __forceinline__ uint4 pack16(const float *f) {
     if constexpr (std::is_same<T, BF16>::value) {
-        if constexpr (EV == 8) {
-            st_stream16(p, make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
-                                      pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7])));
-        } else {
-            st_stream8(p, make_uint2(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3])));
-        }
+        return make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
+                          pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
     } else {
-        st_stream16(p, make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]),
-                                  __float_as_uint(f[2]), __float_as_uint(f[3])));
-        if constexpr (EV == 8) {
-            st_stream16(p + 16, make_uint4(__float_as_uint(f[4]), __float_as_uint(f[5]),
-                                           __float_as_uint(f[6]), __float_as_uint(f[7])));
-        }
+        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                          __float_as_uint(f[3]));
+    }
+}
+
+// N consecutive elements of T at byte address p, N * sizeof(T) = 8 or a multiple of 16.
+// Addresses are 16-byte aligned (8 for the 8-byte case): outputs and the Euler state are
+// only guaranteed 16-byte alignment, so wider accesses are never used on them.
+template <class T, int N>
+__device__ __forceinline__ void load_plain(const char *p, float *f) {
+    constexpr int B = N * T::kBytes;
+    if constexpr (B == 8) {
+        static_assert(std::is_same<T, BF16>::value, "8-byte groups are 4 bf16");
+        const uint2 r = ld_plain8(p);
+        f[0] = bf16_lo(r.x); f[1] = bf16_hi(r.x); f[2] = bf16_lo(r.y); f[3] = bf16_hi(r.y);
+    } else {
+#pragma unroll
+        for (int q = 0; q < B / 16; ++q) unpack16<T>(ld_plain16(p + 16 * q), f + q * (16 / T::kBytes));
+    }
+}
+
+template <class T, int N>
+__device__ __forceinline__ void store_stream(char *p, const float *f) {
+    constexpr int B = N * T::kBytes;
+    if constexpr (B == 8) {
+        static_assert(std::is_same<T, BF16>::value, "8-byte groups are 4 bf16");
+        st_stream8(p, make_uint2(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3])));
+    } else {
+#pragma unroll
+        for (int q = 0; q < B / 16; ++q) st_stream16(p + 16 * q, pack16<T>(f + q * (16 / T::kBytes)));
     }
 }
 
@@ -175,7 +223,11 @@ __device__ __forceinline__ void seek_layer(const ForecastArgs<CAP> &a, int64_t t
 template <int K, class TIn, class TOut, int CAP>
 __global__ void __launch_bounds__(kThreads)
     forecast_kernel(const __grid_constant__ ForecastArgs<CAP> a) {
-    constexpr int EV = 16 / TIn::kBytes;  // elements per 16-byte history vector
+    constexpr int kVecsPerThread = kVecsPerThreadFor<K>;
+    constexpr int kTileVecs = kThreads * kVecsPerThread;
+    constexpr int EV = kVecBytes / TIn::kBytes;  // elements per history vector
+    constexpr int EV16 = 16 / TIn::kBytes;       // elements per 16-byte piece
+    const uint64_t pol = history_policy();
     float w[K];
 #pragma unroll
     for (int j = 0; j < K; ++j) w[j] = a.w[j];
@@ -195,13 +247,13 @@ __global__ void __launch_bounds__(kThreads)
         const bool euler = (l == a.euler_layer);
 
         // Issue every load of the tile before using any of them.
-        uint4 r[kVecsPerThread][K];
+        Raw r[kVecsPerThread][K];
 #pragma unroll
         for (int u = 0; u < kVecsPerThread; ++u) {
             const int64_t v = v0 + u * kThreads;
             if (v < nvec) {
 #pragma unroll
-                for (int j = 0; j < K; ++j) r[u][j] = ld_stream16(src[j] + v * 16);
+                for (int j = 0; j < K; ++j) r[u][j] = ld_history(src[j] + v * kVecBytes, pol);
             }
         }
 #pragma unroll
@@ -209,31 +261,34 @@ __global__ void __launch_bounds__(kThreads)
             const int64_t v = v0 + u * kThreads;
             if (v < nvec) {
                 float acc[EV], f[EV];
-                unpack16<TIn>(r[u][0], f);
+#pragma unroll
+                for (int q = 0; q < kVecBytes / 16; ++q) unpack16<TIn>(r[u][0].q[q], f + q * EV16);
 #pragma unroll
                 for (int e = 0; e < EV; ++e) acc[e] = w[0] * f[e];
 #pragma unroll
                 for (int j = 1; j < K; ++j) {
-                    unpack16<TIn>(r[u][j], f);
+#pragma unroll
+                    for (int q = 0; q < kVecBytes / 16; ++q)
+                        unpack16<TIn>(r[u][j].q[q], f + q * EV16);
 #pragma unroll
                     for (int e = 0; e < EV; ++e) acc[e] = fmaf(w[j], f[e], acc[e]);
                 }
-                if (!euler) {
-                    store_elems<TOut, EV>(dst, v * EV, acc);
-                } else {
-                    if (dst) store_elems<TOut, EV>(dst, v * EV, acc);
+                if (dst) store_stream<TOut, EV>(dst + v * EV * TOut::kBytes, acc);
+                if (euler) {
                     float x[EV];
-                    char *xb = reinterpret_cast<char *>(a.x);
+                    char *xp = reinterpret_cast<char *>(a.x);
                     if (a.x_bf16) {
-                        load_elems<BF16, EV>(xb, v * EV, x);
+                        xp += v * EV * 2;
+                        load_plain<BF16, EV>(xp, x);
 #pragma unroll
                         for (int e = 0; e < EV; ++e) x[e] = fmaf(a.dt, acc[e], x[e]);
-                        store_elems<BF16, EV>(xb, v * EV, x);
+                        store_stream<BF16, EV>(xp, x);
                     } else {
-                        load_elems<F32, EV>(xb, v * EV, x);
+                        xp += v * EV * 4;
+                        load_plain<F32, EV>(xp, x);
 #pragma unroll
                         for (int e = 0; e < EV; ++e) x[e] = fmaf(a.dt, acc[e], x[e]);
-                        store_elems<F32, EV>(xb, v * EV, x);
+                        store_stream<F32, EV>(xp, x);
                     }
                 }
             }
@@ -245,10 +300,8 @@ __global__ void __launch_bounds__(kThreads)
             float acc = w[0] * load_scalar<TIn>(src[0], e);
 #pragma unroll
             for (int j = 1; j < K; ++j) acc = fmaf(w[j], load_scalar<TIn>(src[j], e), acc);
-            if (!euler) {
-                store_scalar<TOut>(dst, e, acc);
-            } else {
-                if (dst) store_scalar<TOut>(dst, e, acc);
+            if (dst) store_scalar<TOut>(dst, e, acc);
+            if (euler) {
                 char *xb = reinterpret_cast<char *>(a.x);
                 if (a.x_bf16)
                     store_scalar<BF16>(xb, e, fmaf(a.dt, acc, load_scalar<BF16>(xb, e)));
@@ -260,8 +313,11 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // Grouped byte-exact copy for the push: layer.src -> layer.dst, numel elements of T.
+// Always 16-byte vectors: the caller's source is only guaranteed 16-byte alignment.
 template <class T, int CAP>
 __global__ void __launch_bounds__(kThreads) copy_kernel(const __grid_constant__ ForecastArgs<CAP> a) {
+    constexpr int kVecsPerThread = kCopyVecsPerThread;
+    constexpr int kTileVecs = kThreads * kVecsPerThread;
     constexpr int EV = 16 / T::kBytes;
     int l = 0;
     int64_t first = 0;
@@ -306,24 +362,28 @@ int sm_count() {
     return g_sm_count;
 }
 
+// Resident CTAs per SM for a kernel, optionally capped (the forecast runs best at two
+// 256-thread CTAs per SM; the single-stream copy at full occupancy).
 template <class KernelPtr>
-int resident_ctas(KernelPtr kern, int &cache) {
+int resident_ctas(KernelPtr kern, int &cache, int cap) {
     if (cache == 0) {
         int n = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, kThreads, 0) != cudaSuccess ||
             n < 1)
             n = 1;
+        if (cap > 0 && cap < n) n = cap;
         cache = n;
     }
     return cache;
 }
 
 template <int CAP>
-int64_t fill_table(ForecastArgs<CAP> &a, const LayerEntry *layers, int n, int elem_bytes) {
+int64_t fill_table(ForecastArgs<CAP> &a, const LayerEntry *layers, int n, int elem_bytes,
+                   int vec_bytes, int tile_vecs) {
     int64_t tiles = 0;
     for (int i = 0; i < n; ++i) {
         a.layer[i] = layers[i];
-        tiles += tiles_for(layers[i].numel, elem_bytes);
+        tiles += tiles_for(layers[i].numel, elem_bytes, vec_bytes, tile_vecs);
         a.layer[i].tile_end = tiles;
     }
     a.n_layers = n;
@@ -344,10 +404,11 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
     a.euler_layer = euler_local;
     a.x_bf16 = p.x_dtype == BC_DTYPE_BF16 ? 1 : 0;
     a.x = p.x;
-    a.total_tiles = fill_table(a, layers, n, TIn::kBytes);
+    a.total_tiles =
+        fill_table(a, layers, n, TIn::kBytes, kVecBytes, kThreads * kVecsPerThreadFor<K>);
     if (a.total_tiles == 0) return cudaSuccess;
     auto kern = forecast_kernel<K, TIn, TOut, CAP>;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ);
+    const int64_t cap = static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ, BC_CTAS_PER_SM);
     const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
     kern<<<grid, kThreads, 0, s>>>(a);
     ++*launches;
@@ -384,10 +445,10 @@ int copy_group(const LayerEntry *layers, int n, cudaStream_t s, int64_t *launche
     ForecastArgs<CAP> a;
     memset(&a, 0, sizeof a);
     a.euler_layer = -1;
-    a.total_tiles = fill_table(a, layers, n, T::kBytes);
+    a.total_tiles = fill_table(a, layers, n, T::kBytes, 16, kThreads * kCopyVecsPerThread);
     if (a.total_tiles == 0) return cudaSuccess;
     auto kern = copy_kernel<T, CAP>;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ);
+    const int64_t cap = static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ, 0);
     const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
     kern<<<grid, kThreads, 0, s>>>(a);
     ++*launches;

@@ -8,11 +8,38 @@
 
 namespace bc {
 
-// Elements of a layer are processed in tiles of kTileVecs 16-byte vectors (kThreads
-// threads x kVecsPerThread vectors); a tile never straddles two layers.
-constexpr int kThreads = 256;
-constexpr int kVecsPerThread = 4;
-constexpr int kTileVecs = kThreads * kVecsPerThread;
+// Tuning constants of the streaming kernels.  They are compile-time so that the compiler
+// unrolls every per-thread loop.  The defaults are the best of a sweep on GB300 (t2v
+// workload, K = 2..4): 32-byte history loads, 256-thread CTAs, two CTAs per SM, two
+// vectors per thread and slot (four at K = 4).  The BC_* macros exist to build variants
+// for tuning sweeps.
+#ifndef BC_VEC_BYTES
+#define BC_VEC_BYTES 32      // bytes per history vector load (16 or 32)
+#endif
+#ifndef BC_VECS_PER_THREAD
+#define BC_VECS_PER_THREAD 0 // 0: per-K default (vecs_per_thread below)
+#endif
+#ifndef BC_THREADS
+#define BC_THREADS 256
+#endif
+#ifndef BC_L2_EVICT_FIRST
+#define BC_L2_EVICT_FIRST 0  // 1: history loads carry an L2 evict-first cache policy
+#endif
+#ifndef BC_CTAS_PER_SM
+#define BC_CTAS_PER_SM 2     // 0: as many as the occupancy calculator allows
+#endif
+
+// Elements of a layer are processed in tiles of kThreads x VPT vectors of kVecBytes
+// (VPT = vectors per thread, per history slot); a tile never straddles two layers.
+constexpr int kVecBytes = BC_VEC_BYTES;
+constexpr int kThreads = BC_THREADS;
+static_assert(kVecBytes == 16 || kVecBytes == 32, "vector loads are 16 or 32 bytes");
+
+// Independent vectors per thread and history slot for a K-term forecast.
+template <int K>
+constexpr int kVecsPerThreadFor = BC_VECS_PER_THREAD > 0 ? BC_VECS_PER_THREAD : (K >= 4 ? 4 : 2);
+// The push copy streams one source: four 16-byte vectors per thread.
+constexpr int kCopyVecsPerThread = 4;
 
 // Layers per launch carried in the kernel's parameter block.  The whole table travels as
 // a __grid_constant__ parameter, so a forecast needs no device-side scratch and no
@@ -56,11 +83,12 @@ struct LaunchPlan {
     int n_layers;
 };
 
-// Tiles needed for `numel` elements of `elem_bytes` each.
-inline int64_t tiles_for(int64_t numel, int elem_bytes) {
-    const int64_t ev = 16 / elem_bytes;
+// Tiles needed for `numel` elements of `elem_bytes` each, in vectors of `vec_bytes`,
+// `tile_vecs` vectors per tile.
+inline int64_t tiles_for(int64_t numel, int elem_bytes, int vec_bytes, int tile_vecs) {
+    const int64_t ev = vec_bytes / elem_bytes;
     const int64_t vecs = (numel + ev - 1) / ev;
-    return (vecs + kTileVecs - 1) / kTileVecs;
+    return (vecs + tile_vecs - 1) / tile_vecs;
 }
 
 // Enqueue the grouped forecast (one launch per CAP-sized group of layers).  Returns the
