@@ -14,6 +14,10 @@ Functions (paper: BaryCache, Sec. 3.2-3.3, Eqs. 8-13):
 * :func:`combine` -- Eq. 13 element by element, with the tolerance scale sum_j |W_j||F_j|.
 * :func:`euler` -- Eq. 13 on the cached velocity followed by x + dt * v_hat.
 * :func:`bf16_to_float64` -- exact widening of stored bf16 words.
+* :func:`ddpm_coefficients` -- Eq. 3's mean and Eq. 2's deviation as x' = a x + b eps + c z.
+* :func:`ddim_coefficients` -- the DDIM step (Song et al., ICLR 2021) in the same form.
+* :func:`update` -- Eq. 13 on the cached model output, then x' = a x + b v_hat + c z.
+* :func:`drift` -- the relative L1 probe drift of the adaptive schedule (Sec. 4.5).
 """
 from __future__ import annotations
 
@@ -74,6 +78,18 @@ def _load():
                                          ctypes.c_double, ctypes.c_int, ctypes.c_void_p,
                                          dp, dp, dp]
             lib.oracle_euler.restype = None
+            d = ctypes.c_double
+            lib.oracle_ddpm_coefficients.argtypes = [d, d, dp, dp, dp]
+            lib.oracle_ddpm_coefficients.restype = ctypes.c_int
+            lib.oracle_ddim_coefficients.argtypes = [d, d, d, dp, dp, dp]
+            lib.oracle_ddim_coefficients.restype = ctypes.c_int
+            lib.oracle_update.argtypes = [ctypes.c_int, vpp, ctypes.c_int, dp, ctypes.c_int64,
+                                          d, d, d, ctypes.c_int, ctypes.c_void_p,
+                                          ctypes.c_void_p, dp, dp]
+            lib.oracle_update.restype = None
+            lib.oracle_drift.argtypes = [ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
+                                         ctypes.c_int64, dp]
+            lib.oracle_drift.restype = None
             _lib = lib
     return _lib
 
@@ -174,3 +190,59 @@ def euler(V: list[np.ndarray], W, x: np.ndarray, dt: float):
                          ctypes.c_void_p(xa.ctypes.data), _dptr(x_new), _dptr(v_hat),
                          _dptr(bound))
     return x_new, v_hat, bound
+
+
+def ddpm_coefficients(alpha_t: float, alpha_bar_t: float) -> tuple[float, float, float]:
+    a, b, c = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    rc = _load().oracle_ddpm_coefficients(alpha_t, alpha_bar_t, ctypes.byref(a),
+                                          ctypes.byref(b), ctypes.byref(c))
+    if rc != OK:
+        raise OracleError(f"oracle_ddpm_coefficients status {rc}")
+    return a.value, b.value, c.value
+
+
+def ddim_coefficients(alpha_bar_t: float, alpha_bar_prev: float,
+                      eta: float = 0.0) -> tuple[float, float, float]:
+    a, b, c = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    rc = _load().oracle_ddim_coefficients(alpha_bar_t, alpha_bar_prev, eta, ctypes.byref(a),
+                                          ctypes.byref(b), ctypes.byref(c))
+    if rc != OK:
+        raise OracleError(f"oracle_ddim_coefficients status {rc}")
+    return a.value, b.value, c.value
+
+
+def update(V: list[np.ndarray], W, x: np.ndarray, a: float, b: float, c: float = 0.0,
+           z: np.ndarray | None = None):
+    """Eq. 13 on the cached model output, then x' = a x + b v_hat + c z.
+
+    Returns (x_new, bound), float64, bound = |a x| + |b| sum_j |W_j||V_j| + |c z|.
+    """
+    W = np.ascontiguousarray(W, dtype=np.float64)
+    m = len(W)
+    arrs = [np.ascontiguousarray(v).reshape(-1) for v in V]
+    code = _dtype_code(arrs[0])
+    xa = np.ascontiguousarray(x).reshape(-1)
+    n = arrs[0].size
+    za = None if z is None else np.ascontiguousarray(z).reshape(-1)
+    if xa.size != n or (za is not None and (za.size != n or za.dtype != xa.dtype)):
+        raise ValueError("x (and z) must match the velocity's size; z has x's dtype")
+    ptrs = (ctypes.c_void_p * m)(*[v.ctypes.data for v in arrs])
+    x_new = np.empty(n, dtype=np.float64)
+    bound = np.empty(n, dtype=np.float64)
+    _load().oracle_update(code, ptrs, m, _dptr(W), n, float(a), float(b), float(c),
+                          _dtype_code(xa), ctypes.c_void_p(xa.ctypes.data),
+                          None if za is None else ctypes.c_void_p(za.ctypes.data),
+                          _dptr(x_new), _dptr(bound))
+    return x_new, bound
+
+
+def drift(cur: np.ndarray, prev: np.ndarray) -> np.ndarray:
+    """[sum |cur - prev|, sum |prev|, ratio] in float64 (Sec. 4.5 probe drift)."""
+    c = np.ascontiguousarray(cur).reshape(-1)
+    p = np.ascontiguousarray(prev).reshape(-1)
+    if c.size != p.size or c.dtype != p.dtype:
+        raise ValueError("cur and prev must match")
+    out = np.zeros(3, dtype=np.float64)
+    _load().oracle_drift(_dtype_code(c), ctypes.c_void_p(c.ctypes.data),
+                         ctypes.c_void_p(p.ctypes.data), c.size, _dptr(out))
+    return out

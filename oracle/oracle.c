@@ -12,7 +12,10 @@
  *     the remark under Eq. 8);
  *   - the paper's stabilised weights, Eqs. 8-12, step by step in the paper's order;
  *   - the weight application of Eq. 13, x_hat = sum_j W_j * x_{f=-j}, element by element;
- *   - the fused Euler update x <- x + dt * x_hat used by the flow-matching sampler (Sec. 4.1).
+ *   - the fused Euler update x <- x + dt * x_hat used by the flow-matching sampler (Sec. 4.1);
+ *   - the DDPM step of Eqs. 2-3, the DDIM step (from the DDIM paper; the sampler the paper
+ *     uses for C2I/T2I, Sec. 4.1) and the general update x <- a x + b x_hat + c z;
+ *   - the relative L1 drift of a feature probe that drives the adaptive schedule (Sec. 4.5).
  *
  * Index convention (Sec. 3.2, "Get Key"): node j = 1 is the most recent cached feature
  * x_{f=-1} with timestep s_1; node H is the oldest.  In C arrays that is index j-1.
@@ -197,4 +200,92 @@ void oracle_euler(int v_dtype, const void *const *V, int m, const double *W, int
         if (v_hat) v_hat[e] = acc;
         if (bound) bound[e] = fabs(x0) + fabs(dt) * mag;
     }
+}
+
+/* ---------------------------------------------------------------------------------
+ * Sampler updates applied to the forecast of the cached model output.
+ *
+ * DDPM reverse step, Sec. 3.1: Eq. 3 gives the mean
+ *     mu = (1 / sqrt(alpha_t)) * (x_t - (1 - alpha_t) / sqrt(1 - alpha_bar_t) * eps)
+ * and Eq. 2 the variance beta_t; beta_t is read as 1 - alpha_t, the noise variance of the
+ * forward step in Eq. 1.  Written as x_{t-1} = a x_t + b eps + c z.
+ * ------------------------------------------------------------------------------- */
+int oracle_ddpm_coefficients(double alpha_t, double alpha_bar_t, double *a, double *b,
+                             double *c)
+{
+    if (!(alpha_t > 0.0 && alpha_t <= 1.0) || !(alpha_bar_t > 0.0 && alpha_bar_t < 1.0))
+        return ORACLE_BAD_ARG;
+    double inv_sqrt_alpha = 1.0 / sqrt(alpha_t);
+    double eps_scale = (1.0 - alpha_t) / sqrt(1.0 - alpha_bar_t);
+    *a = inv_sqrt_alpha;
+    *b = -inv_sqrt_alpha * eps_scale;
+    *c = sqrt(1.0 - alpha_t);
+    return ORACLE_OK;
+}
+
+/* DDIM (Song, Meng, Ermon, ICLR 2021): the paper's C2I/T2I sampler (Sec. 4.1) is not
+ * printed in it, so this follows the DDIM paper's generative step from alpha_bar_t to
+ * alpha_bar_prev:
+ *     x0_pred = (x_t - sqrt(1 - alpha_bar_t) eps) / sqrt(alpha_bar_t)
+ *     x_prev  = sqrt(alpha_bar_prev) x0_pred + sqrt(1 - alpha_bar_prev - sigma^2) eps
+ *               + sigma z
+ *     sigma   = eta sqrt((1 - alpha_bar_prev) / (1 - alpha_bar_t))
+ *                   sqrt(1 - alpha_bar_t / alpha_bar_prev)
+ * collected as x_prev = a x_t + b eps + c z. */
+int oracle_ddim_coefficients(double alpha_bar_t, double alpha_bar_prev, double eta, double *a,
+                             double *b, double *c)
+{
+    if (!(alpha_bar_t > 0.0 && alpha_bar_t < 1.0) ||
+        !(alpha_bar_prev >= alpha_bar_t && alpha_bar_prev <= 1.0) || !(eta >= 0.0))
+        return ORACLE_BAD_ARG;
+    double sigma = eta * sqrt((1.0 - alpha_bar_prev) / (1.0 - alpha_bar_t)) *
+                   sqrt(1.0 - alpha_bar_t / alpha_bar_prev);
+    double dir_var = 1.0 - alpha_bar_prev - sigma * sigma;
+    if (dir_var < 0.0) return ORACLE_BAD_ARG;
+    /* x0_pred contributes sqrt(abp)/sqrt(abt) * x_t and -sqrt(abp) sqrt(1-abt)/sqrt(abt) * eps */
+    double x0_from_x = 1.0 / sqrt(alpha_bar_t);
+    double x0_from_eps = -sqrt(1.0 - alpha_bar_t) / sqrt(alpha_bar_t);
+    *a = sqrt(alpha_bar_prev) * x0_from_x;
+    *b = sqrt(alpha_bar_prev) * x0_from_eps + sqrt(dir_var);
+    *c = sigma;
+    return ORACLE_OK;
+}
+
+/* Forecast of the cached model output followed by x <- a x + b v_hat + c z.  z may be NULL
+ * (no noise term); x and z are stored in x_dtype.  bound[e] = |a x| + |b| sum_j |W_j||V_j|
+ * + |c z|. */
+void oracle_update(int v_dtype, const void *const *V, int m, const double *W, int64_t n,
+                   double a, double b, double c, int x_dtype, const void *x, const void *z,
+                   double *x_out, double *bound)
+{
+    for (int64_t e = 0; e < n; ++e) {
+        double acc = 0.0, mag = 0.0;
+        for (int j = 0; j < m; ++j) {
+            double v = load_elem(v_dtype, V[j], e);
+            acc += W[j] * v;
+            mag += fabs(W[j]) * fabs(v);
+        }
+        double x0 = load_elem(x_dtype, x, e);
+        double z0 = z ? load_elem(x_dtype, z, e) : 0.0;
+        x_out[e] = a * x0 + b * acc + c * z0;
+        if (bound) bound[e] = fabs(a * x0) + fabs(b) * mag + fabs(c * z0);
+    }
+}
+
+/* ---------------------------------------------------------------------------------
+ * Feature-probe drift of the adaptive schedule (Sec. 4.5): the relative L1 change
+ *     out[0] = sum |cur - prev|,  out[1] = sum |prev|,  out[2] = out[0] / out[1]
+ * (0 when both sums vanish, +inf when only the denominator does).
+ * ------------------------------------------------------------------------------- */
+void oracle_drift(int dtype, const void *cur, const void *prev, int64_t n, double *out)
+{
+    double num = 0.0, den = 0.0;
+    for (int64_t e = 0; e < n; ++e) {
+        double c = load_elem(dtype, cur, e), p = load_elem(dtype, prev, e);
+        num += fabs(c - p);
+        den += fabs(p);
+    }
+    out[0] = num;
+    out[1] = den;
+    out[2] = den > 0.0 ? num / den : (num > 0.0 ? INFINITY : 0.0);
 }
