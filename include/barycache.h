@@ -78,7 +78,7 @@ typedef struct {
 typedef struct bc_cache *bc_handle;
 
 typedef struct {
-    int64_t forecasts;       /* successful bc_forecast / bc_forecast_step calls */
+    int64_t forecasts;       /* successful forecast calls (every bc_forecast* variant) */
     int64_t pushes;          /* successful bc_cache_push / bc_cache_commit calls */
     int64_t kernel_launches; /* CUDA kernels this handle has launched */
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
@@ -117,17 +117,19 @@ bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtyp
 /* ------------------------------------------------------------ cache lifecycle */
 
 /* Create the cache context H_t of Eq. 6 for `n_layers` tensors of numels[l] elements of
- * `dtype`, with history length K (1..BC_MAX_K).  Allocates one device arena of
- * bc_cache_bytes_for(...) bytes on the current device (the only device allocation the
- * library makes; freed by bc_cache_destroy).  p == NULL uses the paper's defaults.
- * Blocks until the allocation is done.  Errors: INVALID_ARG, OOM, CUDA. */
+ * `dtype`, with history length K (1..BC_MAX_K).  Allocates, on the current device, one
+ * arena of bc_cache_bytes_for(...) bytes and 16 KiB of reduction scratch for
+ * bc_probe_drift (the only device allocations the library makes; freed by
+ * bc_cache_destroy).  p == NULL uses the paper's defaults.  Blocks until the allocation is
+ * done.  Errors: INVALID_ARG, OOM, CUDA. */
 bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
                           const bc_params *p, bc_handle *out);
 
 /* Free the arena (synchronises the device first so no enqueued work still reads it). */
 bc_status bc_cache_destroy(bc_handle h);
 
-/* Device bytes held by this cache (arena only; host bookkeeping is not counted). */
+/* Device bytes held by this cache: the arena (the 16 KiB reduction scratch and host
+ * bookkeeping are not counted). */
 bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
 
 /* Replace the weight parameters (clears the weight memo). */
@@ -187,6 +189,86 @@ bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype
 bc_status bc_forecast_step(bc_handle h, double t_new, double dt, void *const *out_ptrs,
                            bc_dtype out_dtype, int v_layer, void *x, bc_dtype x_dtype,
                            void *stream);
+
+/* Forecast fused with a general sampler update on layer `v_layer` (the cached model output,
+ * e.g. the noise prediction eps of Eq. 3 or a flow velocity), in the same launch as the
+ * forecast of every other selected layer:
+ *     v_hat[e] = sum_j W_j V_j[e],    x[e] <- a x[e] + b v_hat[e] + c z[e]   (fp32 math)
+ * z (device, numels[v_layer] elements of x_dtype, 16-byte aligned, read only) may be NULL
+ * (no noise term).  Coefficients for the DDPM mean of Eq. 3 and for DDIM come from
+ * bc_ddpm_coefficients / bc_ddim_coefficients; Euler is a = 1, b = dt, c = 0
+ * (bc_forecast_step).  x and z must not overlap each other, an output or the arena.
+ * Errors as bc_forecast_step (INVALID_ARG also for non-finite coefficients). */
+bc_status bc_forecast_update(bc_handle h, double t_new, double a, double b, double c,
+                             void *const *out_ptrs, bc_dtype out_dtype, int v_layer, void *x,
+                             bc_dtype x_dtype, const void *z, void *stream);
+
+/* Skipped-step forecast of every layer into one output buffer laid out like a cache slot:
+ * layer l's forecast starts at byte offset offsets[l] of bc_cache_layout, in the cache
+ * dtype.  One launch whatever the number of layers (the many-tensor blockwise layout of
+ * Sec. 4.5, Tables 5-6), with no per-layer table.  `out` (device, 16-byte aligned,
+ * offsets[n_layers] bytes) must not overlap the arena.  The padding between layers is
+ * written with unspecified values.  Errors as bc_forecast. */
+bc_status bc_forecast_flat(bc_handle h, double t_new, void *out, void *stream);
+
+/* Byte offset of every layer inside a slot (and inside a bc_forecast_flat output), in
+ * offsets[0 .. n_layers-1]; offsets[n_layers] = bytes per slot. */
+bc_status bc_cache_layout(bc_handle h, int64_t *offsets);
+
+/* ------------------------------------------------------------ sampler coefficients */
+
+/* DDPM reverse step (Sec. 3.1, Eqs. 2-3) as x_{t-1} = a x_t + b eps + c z:
+ * a = 1/sqrt(alpha_t), b = -(1 - alpha_t) / (sqrt(alpha_t) sqrt(1 - alpha_bar_t)), and the
+ * Eq. 2 standard deviation c = sqrt(beta_t) with beta_t = 1 - alpha_t (the noise scale of
+ * Eq. 1).  Needs 0 < alpha_t <= 1, 0 < alpha_bar_t < 1.  Host only. */
+bc_status bc_ddpm_coefficients(double alpha_t, double alpha_bar_t, double *a, double *b,
+                               double *c);
+
+/* DDIM step (Song, Meng and Ermon, "Denoising Diffusion Implicit Models", ICLR 2021; the
+ * paper's C2I/T2I sampler, Sec. 4.1) from alpha_bar_t to alpha_bar_prev with parameter eta
+ * (0 = deterministic), as x_prev = a x_t + b eps + c z:
+ *   sigma = eta sqrt((1 - ab_prev)/(1 - ab_t)) sqrt(1 - ab_t/ab_prev),
+ *   a = sqrt(ab_prev/ab_t), b = sqrt(1 - ab_prev - sigma^2) - sqrt(ab_prev (1 - ab_t)/ab_t),
+ *   c = sigma.
+ * Needs 0 < ab_t < 1, ab_t <= ab_prev <= 1, eta >= 0 with 1 - ab_prev - sigma^2 >= 0. */
+bc_status bc_ddim_coefficients(double alpha_bar_t, double alpha_bar_prev, double eta, double *a,
+                               double *b, double *c);
+
+/* ------------------------------------------------------------ schedules (Sec. 3.3, 4.5) */
+
+/* Equal-spaced schedule: is_full[i] = 1 when step i runs the full model, i.e. i < K (the
+ * window fills) or i mod interval == 0; 0 when it is a cache forward.  With K = 2 this
+ * gives ceil(n/interval) + 1 full steps, the count implied by the FLOPs of Tables 1 and 3.
+ * Host only. */
+bc_status bc_schedule_equal(int n_steps, int interval, int K, uint8_t *is_full);
+
+/* Adaptive schedule (Sec. 4.5, Table 5): the relative change of a feature probe between
+ * consecutive steps is accumulated and a full step is run once the sum reaches
+ * `threshold` (the paper's l), after which the sum restarts at 0.  The first K steps are
+ * full (the window fills).  Host-only state, one per sampling run. */
+typedef struct {
+    double threshold;    /* l */
+    double accumulated;  /* drift accumulated since the last full step */
+    int32_t K;           /* warm-up full steps */
+    int32_t steps;       /* decisions taken */
+    int32_t full_steps;  /* of which full */
+} bc_adaptive;
+
+bc_status bc_adaptive_init(bc_adaptive *s, double threshold, int K);
+
+/* Decide the next step from its probe drift (>= 0; pass 0 when there is no previous
+ * probe): *run_full = 1 for a full step, 0 for a cache forward. */
+bc_status bc_adaptive_decide(bc_adaptive *s, double drift, int *run_full);
+
+/* The probe drift of the adaptive schedule, on the device:
+ *     out[0] = sum_e |cur[e] - prev[e]|,  out[1] = sum_e |prev[e]|,  out[2] = out[0]/out[1]
+ * (out[2] = 0 when both sums are 0, +inf when only out[1] is).  cur, prev: device, n
+ * elements of dtype, 16-byte aligned; out: 3 device doubles.  Two launches on `stream` with
+ * a fixed reduction order (bitwise reproducible on one device), using the handle's
+ * reduction scratch, so calls on one handle must not overlap on the device.  The caller
+ * reads out[2] back to drive bc_adaptive_decide.  Errors: INVALID_ARG, ALIGNMENT, CUDA. */
+bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
+                         bc_dtype dtype, double *out, void *stream);
 
 /* Counters of this handle (see bc_stats). */
 bc_status bc_cache_stats(bc_handle h, bc_stats *out);

@@ -35,6 +35,11 @@ class bc_params(ctypes.Structure):
                 ("eta", ctypes.c_double)]
 
 
+class bc_adaptive(ctypes.Structure):
+    _fields_ = [("threshold", ctypes.c_double), ("accumulated", ctypes.c_double),
+                ("K", ctypes.c_int32), ("steps", ctypes.c_int32), ("full_steps", ctypes.c_int32)]
+
+
 class bc_stats(ctypes.Structure):
     _fields_ = [("forecasts", ctypes.c_int64), ("pushes", ctypes.c_int64),
                 ("kernel_launches", ctypes.c_int64), ("memo_hits", ctypes.c_int64),
@@ -77,6 +82,26 @@ _SIGNATURES = {
                           ctypes.POINTER(ctypes.c_void_p), ctypes.c_int, ctypes.c_int,
                           ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p], ctypes.c_int),
     "bc_cache_stats": ([ctypes.c_void_p, ctypes.POINTER(bc_stats)], ctypes.c_int),
+    "bc_forecast_update": ([ctypes.c_void_p, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                            ctypes.c_double, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int,
+                            ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+                            ctypes.c_void_p], ctypes.c_int),
+    "bc_forecast_flat": ([ctypes.c_void_p, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p],
+                         ctypes.c_int),
+    "bc_cache_layout": ([ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)], ctypes.c_int),
+    "bc_ddpm_coefficients": ([ctypes.c_double, ctypes.c_double, ctypes.POINTER(ctypes.c_double),
+                              ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)],
+                             ctypes.c_int),
+    "bc_ddim_coefficients": ([ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                              ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                              ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+    "bc_schedule_equal": ([ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                           ctypes.POINTER(ctypes.c_uint8)], ctypes.c_int),
+    "bc_adaptive_init": ([ctypes.c_void_p, ctypes.c_double, ctypes.c_int], ctypes.c_int),
+    "bc_adaptive_decide": ([ctypes.c_void_p, ctypes.c_double, ctypes.POINTER(ctypes.c_int)],
+                           ctypes.c_int),
+    "bc_probe_drift": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                        ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p], ctypes.c_int),
 }
 
 
@@ -234,3 +259,63 @@ def bc_cache_stats(h: int) -> dict:
     s = bc_stats()
     _check(lib().bc_cache_stats(h, ctypes.byref(s)), "bc_cache_stats")
     return {k: getattr(s, k) for k, _ in bc_stats._fields_}
+
+
+def bc_forecast_update(h: int, t_new: float, a: float, b: float, c: float,
+                       out_ptrs: Sequence[int | None], out_dtype: int, v_layer: int, x: int,
+                       x_dtype: int, z: int | None = None, stream: int = 0) -> None:
+    _check(lib().bc_forecast_update(h, float(t_new), float(a), float(b), float(c),
+                                    _ptr_array(out_ptrs), out_dtype, v_layer, x or None,
+                                    x_dtype, z or None, stream or None), "bc_forecast_update")
+
+
+def bc_forecast_flat(h: int, t_new: float, out: int, stream: int = 0) -> None:
+    _check(lib().bc_forecast_flat(h, float(t_new), out or None, stream or None),
+           "bc_forecast_flat")
+
+
+def bc_cache_layout(h: int, n_layers: int) -> list[int]:
+    out = (ctypes.c_int64 * (n_layers + 1))()
+    _check(lib().bc_cache_layout(h, out), "bc_cache_layout")
+    return list(out)
+
+
+def bc_ddpm_coefficients(alpha_t: float, alpha_bar_t: float) -> tuple[float, float, float]:
+    a, b, c = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    _check(lib().bc_ddpm_coefficients(float(alpha_t), float(alpha_bar_t), ctypes.byref(a),
+                                      ctypes.byref(b), ctypes.byref(c)), "bc_ddpm_coefficients")
+    return a.value, b.value, c.value
+
+
+def bc_ddim_coefficients(alpha_bar_t: float, alpha_bar_prev: float,
+                         eta: float = 0.0) -> tuple[float, float, float]:
+    a, b, c = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    _check(lib().bc_ddim_coefficients(float(alpha_bar_t), float(alpha_bar_prev), float(eta),
+                                      ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)),
+           "bc_ddim_coefficients")
+    return a.value, b.value, c.value
+
+
+def bc_schedule_equal(n_steps: int, interval: int, K: int) -> list[int]:
+    out = (ctypes.c_uint8 * max(n_steps, 1))()
+    _check(lib().bc_schedule_equal(n_steps, interval, K, out), "bc_schedule_equal")
+    return list(out[:n_steps])
+
+
+def bc_adaptive_init(threshold: float, K: int) -> bc_adaptive:
+    st = bc_adaptive()
+    _check(lib().bc_adaptive_init(ctypes.byref(st), float(threshold), K), "bc_adaptive_init")
+    return st
+
+
+def bc_adaptive_decide(st: bc_adaptive, drift: float) -> int:
+    full = ctypes.c_int()
+    _check(lib().bc_adaptive_decide(ctypes.byref(st), float(drift), ctypes.byref(full)),
+           "bc_adaptive_decide")
+    return full.value
+
+
+def bc_probe_drift(h: int, cur: int, prev: int, n: int, dtype: int, out: int,
+                   stream: int = 0) -> None:
+    _check(lib().bc_probe_drift(h, cur or None, prev or None, n, dtype, out or None,
+                                stream or None), "bc_probe_drift")

@@ -29,7 +29,7 @@ COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fno-fast-math"
           "-I", INCLUDE, "-I", CSRC]
 
 LIBS = {
-    "libbarycache.so": ["bc_host.cpp", "bc_forecast.cu"],
+    "libbarycache.so": ["bc_host.cpp", "bc_forecast.cu", "bc_probe.cu"],
     "libbc_synth.so": ["bc_synth.cu"],
 }
 HEADERS = [os.path.join(INCLUDE, "barycache.h"), os.path.join(CSRC, "bc_internal.h")]

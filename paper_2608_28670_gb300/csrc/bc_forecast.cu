@@ -275,19 +275,33 @@ __global__ void __launch_bounds__(kThreads)
                 }
                 if (dst) store_stream<TOut, EV>(dst + v * EV * TOut::kBytes, acc);
                 if (euler) {
+                    // Sampler update on the same elements: x <- ca x + cb v_hat (+ cc z).
                     float x[EV];
                     char *xp = reinterpret_cast<char *>(a.x);
+                    const char *zp = reinterpret_cast<const char *>(a.z);
                     if (a.x_bf16) {
                         xp += v * EV * 2;
                         load_plain<BF16, EV>(xp, x);
 #pragma unroll
-                        for (int e = 0; e < EV; ++e) x[e] = fmaf(a.dt, acc[e], x[e]);
+                        for (int e = 0; e < EV; ++e) x[e] = fmaf(a.cb, acc[e], a.ca * x[e]);
+                        if (zp) {
+                            float z[EV];
+                            load_plain<BF16, EV>(zp + v * EV * 2, z);
+#pragma unroll
+                            for (int e = 0; e < EV; ++e) x[e] = fmaf(a.cc, z[e], x[e]);
+                        }
                         store_stream<BF16, EV>(xp, x);
                     } else {
                         xp += v * EV * 4;
                         load_plain<F32, EV>(xp, x);
 #pragma unroll
-                        for (int e = 0; e < EV; ++e) x[e] = fmaf(a.dt, acc[e], x[e]);
+                        for (int e = 0; e < EV; ++e) x[e] = fmaf(a.cb, acc[e], a.ca * x[e]);
+                        if (zp) {
+                            float z[EV];
+                            load_plain<F32, EV>(zp + v * EV * 4, z);
+#pragma unroll
+                            for (int e = 0; e < EV; ++e) x[e] = fmaf(a.cc, z[e], x[e]);
+                        }
                         store_stream<F32, EV>(xp, x);
                     }
                 }
@@ -303,10 +317,16 @@ __global__ void __launch_bounds__(kThreads)
             if (dst) store_scalar<TOut>(dst, e, acc);
             if (euler) {
                 char *xb = reinterpret_cast<char *>(a.x);
-                if (a.x_bf16)
-                    store_scalar<BF16>(xb, e, fmaf(a.dt, acc, load_scalar<BF16>(xb, e)));
-                else
-                    store_scalar<F32>(xb, e, fmaf(a.dt, acc, load_scalar<F32>(xb, e)));
+                const char *zb = reinterpret_cast<const char *>(a.z);
+                if (a.x_bf16) {
+                    float xn = fmaf(a.cb, acc, a.ca * load_scalar<BF16>(xb, e));
+                    if (zb) xn = fmaf(a.cc, load_scalar<BF16>(zb, e), xn);
+                    store_scalar<BF16>(xb, e, xn);
+                } else {
+                    float xn = fmaf(a.cb, acc, a.ca * load_scalar<F32>(xb, e));
+                    if (zb) xn = fmaf(a.cc, load_scalar<F32>(zb, e), xn);
+                    store_scalar<F32>(xb, e, xn);
+                }
             }
         }
     }
@@ -400,7 +420,10 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         a.slot[j] = p.slot[j];
         a.w[j] = p.w[j];
     }
-    a.dt = p.dt;
+    a.ca = p.ca;
+    a.cb = p.cb;
+    a.cc = p.cc;
+    a.z = p.z;
     a.euler_layer = euler_local;
     a.x_bf16 = p.x_dtype == BC_DTYPE_BF16 ? 1 : 0;
     a.x = p.x;

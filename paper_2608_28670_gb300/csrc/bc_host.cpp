@@ -214,6 +214,7 @@ struct bc_cache {
     Memo memo;
     bc_stats stats{};
     std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
+    double *probe_partials = nullptr;             // device scratch of bc_probe_drift
 
     char *slot_base(int slot) const { return arena + static_cast<uint64_t>(slot) * slot_bytes; }
     int slot_of_node(int j) const { return ((head - j) % K + K) % K; }  // j = 0 newest
@@ -265,9 +266,24 @@ void rotate_in(bc_cache *h, double t) {
     ++h->stats.pushes;
 }
 
-bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_ptrs,
-                        bc_dtype out_dtype, int v_layer, void *x, bc_dtype x_dtype,
-                        void *stream) {
+// Sampler update applied to one layer in the forecast's launch: x <- ca x + cb v_hat + cc z.
+struct Update {
+    double ca = 1.0, cb = 0.0, cc = 0.0;
+    int v_layer = -1;
+    void *x = nullptr;
+    bc_dtype x_dtype = BC_DTYPE_F32;
+    const void *z = nullptr;
+};
+
+bool ranges_overlap(uint64_t a, uint64_t an, uint64_t b, uint64_t bn) {
+    return an && bn && a < b + bn && b < a + an;
+}
+
+bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
+                        const Update &up, void *stream) {
+    const int v_layer = up.v_layer;
+    void *x = up.x;
+    const bc_dtype x_dtype = up.x_dtype;
     bc_status s = check_handle(h);
     if (s != BC_OK) return s;
     if (!out_ptrs) return fail(BC_ERR_INVALID_ARG, "out_ptrs is NULL");
@@ -278,7 +294,9 @@ bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_p
         if (!x) return fail(BC_ERR_INVALID_ARG, "x is NULL");
         if (!dtype_valid(x_dtype)) return fail(BC_ERR_INVALID_ARG, "unknown x dtype");
         if (!aligned16(x)) return fail(BC_ERR_ALIGNMENT, "x is not 16-byte aligned");
-        if (!std::isfinite(dt)) return fail(BC_ERR_INVALID_ARG, "non-finite dt");
+        if (up.z && !aligned16(up.z)) return fail(BC_ERR_ALIGNMENT, "z is not 16-byte aligned");
+        if (!std::isfinite(up.ca) || !std::isfinite(up.cb) || !std::isfinite(up.cc))
+            return fail(BC_ERR_INVALID_ARG, "non-finite update coefficient");
     }
     double c[BC_MAX_K];
     int m = 0;
@@ -291,6 +309,9 @@ bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_p
     const uint64_t x0 = reinterpret_cast<uint64_t>(x);
     if (euler && h->overlaps_arena(x0, x_bytes))
         return fail(BC_ERR_INVALID_ARG, "x overlaps the cache arena");
+    const uint64_t z0 = reinterpret_cast<uint64_t>(up.z);
+    if (euler && up.z && (h->overlaps_arena(z0, x_bytes) || ranges_overlap(z0, x_bytes, x0, x_bytes)))
+        return fail(BC_ERR_INVALID_ARG, "z overlaps the cache arena or x");
 
     auto &entries = h->scratch_entries;
     entries.clear();
@@ -304,8 +325,10 @@ bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_p
             const uint64_t p = reinterpret_cast<uint64_t>(o);
             if (h->overlaps_arena(p, ob))
                 return fail(BC_ERR_INVALID_ARG, "output %d overlaps the cache arena", l);
-            if (euler && x_bytes && ob && p < x0 + x_bytes && x0 < p + ob)
+            if (euler && ranges_overlap(p, ob, x0, x_bytes))
                 return fail(BC_ERR_INVALID_ARG, "output %d aliases x", l);
+            if (euler && up.z && ranges_overlap(p, ob, z0, x_bytes))
+                return fail(BC_ERR_INVALID_ARG, "output %d aliases z", l);
         }
         if (euler && l == v_layer) euler_index = static_cast<int>(entries.size());
         bc::LayerEntry e{};
@@ -323,10 +346,13 @@ bc_status forecast_impl(bc_handle h, double t_new, double dt, void *const *out_p
     plan.K = m;
     plan.in_dtype = h->dtype;
     plan.out_dtype = out_dtype;
-    plan.dt = static_cast<float>(dt);
+    plan.ca = static_cast<float>(up.ca);
+    plan.cb = static_cast<float>(up.cb);
+    plan.cc = static_cast<float>(up.cc);
     plan.euler_layer = euler_index;
     plan.x_dtype = x_dtype;
     plan.x = x0;
+    plan.z = up.z ? z0 : 0;
     plan.layers = entries.data();
     plan.n_layers = static_cast<int>(entries.size());
 
@@ -454,6 +480,18 @@ bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype d
             h->arena = static_cast<char *>(mem);
         }
         {
+            void *mem = nullptr;
+            cudaError_t e = cudaMalloc(&mem, sizeof(double) * 2 * bc::kProbeMaxCtas);
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                if (h->arena) cudaFree(h->arena);
+                delete h;
+                return e == cudaErrorMemoryAllocation ? fail(BC_ERR_OOM, "probe scratch")
+                                                      : cuda_fail(e, "cudaMalloc");
+            }
+            h->probe_partials = static_cast<double *>(mem);
+        }
+        {
             std::lock_guard<std::mutex> lk(g_registry_mu);
             g_registry.insert(h);
         }
@@ -478,10 +516,11 @@ bc_status bc_cache_destroy(bc_handle h) {
     }
     h->magic = 0;
     bc_status rc = BC_OK;
-    if (h->arena) {
+    if (h->arena || h->probe_partials) {
         DeviceGuard g(h->device);
         cudaError_t e = cudaDeviceSynchronize();
-        if (e == cudaSuccess) e = cudaFree(h->arena);
+        if (e == cudaSuccess && h->arena) e = cudaFree(h->arena);
+        if (e == cudaSuccess && h->probe_partials) e = cudaFree(h->probe_partials);
         if (e != cudaSuccess) rc = cuda_fail(e, "cudaFree");
     }
     delete h;
@@ -618,8 +657,7 @@ bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype
                       void *stream) {
     t_last_error.clear();
     try {
-        return forecast_impl(h, t_new, 0.0, out_ptrs, out_dtype, -1, nullptr, BC_DTYPE_F32,
-                             stream);
+        return forecast_impl(h, t_new, out_ptrs, out_dtype, Update{}, stream);
     } catch (...) {
         return fail(BC_ERR_INVALID_ARG, "internal exception");
     }
@@ -631,10 +669,188 @@ bc_status bc_forecast_step(bc_handle h, double t_new, double dt, void *const *ou
     t_last_error.clear();
     try {
         if (v_layer < 0) return fail(BC_ERR_INVALID_ARG, "v_layer must name a cached layer");
-        return forecast_impl(h, t_new, dt, out_ptrs, out_dtype, v_layer, x, x_dtype, stream);
+        if (!std::isfinite(dt)) return fail(BC_ERR_INVALID_ARG, "non-finite dt");
+        Update up;
+        up.ca = 1.0;
+        up.cb = dt;
+        up.v_layer = v_layer;
+        up.x = x;
+        up.x_dtype = x_dtype;
+        return forecast_impl(h, t_new, out_ptrs, out_dtype, up, stream);
     } catch (...) {
         return fail(BC_ERR_INVALID_ARG, "internal exception");
     }
+}
+
+bc_status bc_forecast_update(bc_handle h, double t_new, double a, double b, double c,
+                             void *const *out_ptrs, bc_dtype out_dtype, int v_layer, void *x,
+                             bc_dtype x_dtype, const void *z, void *stream) {
+    t_last_error.clear();
+    try {
+        if (v_layer < 0) return fail(BC_ERR_INVALID_ARG, "v_layer must name a cached layer");
+        Update up;
+        up.ca = a;
+        up.cb = b;
+        up.cc = c;
+        up.v_layer = v_layer;
+        up.x = x;
+        up.x_dtype = x_dtype;
+        up.z = z;
+        return forecast_impl(h, t_new, out_ptrs, out_dtype, up, stream);
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_ddpm_coefficients(double alpha_t, double alpha_bar_t, double *a, double *b,
+                               double *c) {
+    t_last_error.clear();
+    if (!a || !b || !c) return fail(BC_ERR_INVALID_ARG, "null pointer");
+    if (!(alpha_t > 0.0 && alpha_t <= 1.0) || !(alpha_bar_t > 0.0 && alpha_bar_t < 1.0))
+        return fail(BC_ERR_INVALID_ARG, "need 0 < alpha_t <= 1 and 0 < alpha_bar_t < 1");
+    // Eq. 3: mu = (x_t - (1 - alpha_t) / sqrt(1 - alpha_bar_t) * eps) / sqrt(alpha_t);
+    // Eq. 2: x_{t-1} ~ N(mu, beta_t I) with beta_t = 1 - alpha_t (the noise scale of Eq. 1).
+    const double ra = std::sqrt(alpha_t);
+    *a = 1.0 / ra;
+    *b = -(1.0 - alpha_t) / (ra * std::sqrt(1.0 - alpha_bar_t));
+    *c = std::sqrt(1.0 - alpha_t);
+    return BC_OK;
+}
+
+bc_status bc_ddim_coefficients(double alpha_bar_t, double alpha_bar_prev, double eta, double *a,
+                               double *b, double *c) {
+    t_last_error.clear();
+    if (!a || !b || !c) return fail(BC_ERR_INVALID_ARG, "null pointer");
+    if (!(alpha_bar_t > 0.0 && alpha_bar_t < 1.0) ||
+        !(alpha_bar_prev >= alpha_bar_t && alpha_bar_prev <= 1.0) || !(eta >= 0.0) ||
+        !std::isfinite(eta))
+        return fail(BC_ERR_INVALID_ARG,
+                    "need 0 < alpha_bar_t < 1, alpha_bar_t <= alpha_bar_prev <= 1, eta >= 0");
+    // DDIM (Song, Meng and Ermon, ICLR 2021, generative process with parameter eta):
+    //   x_prev = sqrt(ab_prev) * (x_t - sqrt(1 - ab_t) eps) / sqrt(ab_t)
+    //            + sqrt(1 - ab_prev - sigma^2) eps + sigma z,
+    //   sigma = eta sqrt((1 - ab_prev) / (1 - ab_t)) sqrt(1 - ab_t / ab_prev).
+    const double sigma = eta * std::sqrt((1.0 - alpha_bar_prev) / (1.0 - alpha_bar_t)) *
+                         std::sqrt(1.0 - alpha_bar_t / alpha_bar_prev);
+    const double dir = 1.0 - alpha_bar_prev - sigma * sigma;
+    if (dir < 0.0) return fail(BC_ERR_INVALID_ARG, "eta too large: negative direction variance");
+    *a = std::sqrt(alpha_bar_prev / alpha_bar_t);
+    *b = std::sqrt(dir) - std::sqrt(alpha_bar_prev * (1.0 - alpha_bar_t) / alpha_bar_t);
+    *c = sigma;
+    return BC_OK;
+}
+
+bc_status bc_cache_layout(bc_handle h, int64_t *offsets) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!offsets) return fail(BC_ERR_INVALID_ARG, "offsets is NULL");
+    for (int l = 0; l < h->n_layers; ++l) offsets[l] = static_cast<int64_t>(h->offset[l]);
+    offsets[h->n_layers] = static_cast<int64_t>(h->slot_bytes);
+    return BC_OK;
+}
+
+bc_status bc_forecast_flat(bc_handle h, double t_new, void *out, void *stream) {
+    t_last_error.clear();
+    try {
+        bc_status s = check_handle(h);
+        if (s != BC_OK) return s;
+        if (!out) return fail(BC_ERR_INVALID_ARG, "out is NULL");
+        if (!aligned16(out)) return fail(BC_ERR_ALIGNMENT, "out is not 16-byte aligned");
+        if (h->overlaps_arena(reinterpret_cast<uint64_t>(out), h->slot_bytes))
+            return fail(BC_ERR_INVALID_ARG, "out overlaps the cache arena");
+        double c[BC_MAX_K];
+        int m = 0;
+        s = window_weights(h, t_new, c, &m);
+        if (s != BC_OK) return s;
+        if (h->slot_bytes > 0) {
+            bc::LayerEntry e{};
+            e.src = 0;
+            e.dst = reinterpret_cast<uint64_t>(out);
+            e.numel = static_cast<int64_t>(h->slot_bytes / elem_bytes(h->dtype));
+            bc::LaunchPlan plan{};
+            for (int j = 0; j < BC_MAX_K; ++j) {
+                plan.slot[j] =
+                    j < m ? reinterpret_cast<uint64_t>(h->slot_base(h->slot_of_node(j))) : 0;
+                plan.w[j] = j < m ? static_cast<float>(c[j]) : 0.0f;
+            }
+            plan.K = m;
+            plan.in_dtype = h->dtype;
+            plan.out_dtype = h->dtype;
+            plan.euler_layer = -1;
+            plan.layers = &e;
+            plan.n_layers = 1;
+            DeviceGuard g(h->device);
+            if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+            const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches);
+            if (err != cudaSuccess) return cuda_fail(err, "forecast launch");
+        }
+        ++h->stats.forecasts;
+        h->stats.memo_hits = h->memo.hits;
+        h->stats.memo_misses = h->memo.misses;
+        return BC_OK;
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
+bc_status bc_schedule_equal(int n_steps, int interval, int K, uint8_t *is_full) {
+    t_last_error.clear();
+    if (n_steps < 0 || interval < 1 || K < 0 || (n_steps > 0 && !is_full))
+        return fail(BC_ERR_INVALID_ARG, "need n_steps >= 0, interval >= 1, K >= 0");
+    for (int i = 0; i < n_steps; ++i) is_full[i] = (i < K || i % interval == 0) ? 1 : 0;
+    return BC_OK;
+}
+
+bc_status bc_adaptive_init(bc_adaptive *st, double threshold, int K) {
+    t_last_error.clear();
+    if (!st) return fail(BC_ERR_INVALID_ARG, "state is NULL");
+    if (!(threshold >= 0.0) || !std::isfinite(threshold) || K < 0)
+        return fail(BC_ERR_INVALID_ARG, "need a finite threshold >= 0 and K >= 0");
+    st->threshold = threshold;
+    st->accumulated = 0.0;
+    st->K = K;
+    st->steps = 0;
+    st->full_steps = 0;
+    return BC_OK;
+}
+
+bc_status bc_adaptive_decide(bc_adaptive *st, double drift, int *run_full) {
+    t_last_error.clear();
+    if (!st || !run_full) return fail(BC_ERR_INVALID_ARG, "null pointer");
+    if (!(drift >= 0.0)) return fail(BC_ERR_INVALID_ARG, "drift must be >= 0 (and not NaN)");
+    int full;
+    if (st->steps < st->K) {
+        full = 1;  // the window is still filling
+    } else {
+        st->accumulated += drift;
+        full = st->accumulated >= st->threshold ? 1 : 0;
+    }
+    if (full) {
+        st->accumulated = 0.0;
+        ++st->full_steps;
+    }
+    ++st->steps;
+    *run_full = full;
+    return BC_OK;
+}
+
+bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
+                         bc_dtype dtype, double *out, void *stream) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (!out || n < 0 || (n > 0 && (!cur || !prev)))
+        return fail(BC_ERR_INVALID_ARG, "need device cur, prev (n elements) and out[3]");
+    if (!dtype_valid(dtype)) return fail(BC_ERR_INVALID_ARG, "unknown dtype");
+    if (!aligned16(cur) || !aligned16(prev))
+        return fail(BC_ERR_ALIGNMENT, "probe tensors must be 16-byte aligned");
+    DeviceGuard g(h->device);
+    if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+    const int err = bc::launch_drift(cur, prev, n, dtype, h->probe_partials, bc::kProbeMaxCtas,
+                                     out, stream, &h->stats.kernel_launches);
+    if (err != cudaSuccess) return cuda_fail(err, "drift launch");
+    return BC_OK;
 }
 
 bc_status bc_cache_stats(bc_handle h, bc_stats *out) {

@@ -59,11 +59,12 @@ template <int CAP>
 struct ForecastArgs {
     uint64_t slot[BC_MAX_K];  // slot base address of node j (j = 0 newest)
     float w[BC_MAX_K];        // weights W_j rounded to fp32
-    float dt;                 // Euler step (only for the Euler layer)
+    float ca, cb, cc;         // sampler update x <- ca x + cb v_hat + cc z (update layer)
     int32_t n_layers;
-    int32_t euler_layer;      // index into `layer`, or -1
-    int32_t x_bf16;           // Euler state dtype: 1 = bf16, 0 = f32
-    uint64_t x;               // Euler state address
+    int32_t euler_layer;      // index into `layer` of the update layer, or -1
+    int32_t x_bf16;           // sampler state dtype (and z's): 1 = bf16, 0 = f32
+    uint64_t x;               // sampler state address
+    uint64_t z;               // noise address (0: no noise term)
     int64_t total_tiles;
     LayerEntry layer[CAP];
 };
@@ -75,10 +76,11 @@ struct LaunchPlan {
     int K;                    // live nodes used (1..BC_MAX_K)
     bc_dtype in_dtype;
     bc_dtype out_dtype;
-    float dt;
+    float ca, cb, cc;
     int euler_layer;          // index into `layers`, or -1
     bc_dtype x_dtype;
     uint64_t x;
+    uint64_t z;
     const LayerEntry *layers; // tile_end filled by the launcher
     int n_layers;
 };
@@ -94,6 +96,14 @@ inline int64_t tiles_for(int64_t numel, int elem_bytes, int vec_bytes, int tile_
 // Enqueue the grouped forecast (one launch per CAP-sized group of layers).  Returns the
 // CUDA error of the last launch; *launches is incremented per launch.
 int launch_forecast(const LaunchPlan &plan, void *stream, int64_t *launches);
+
+// Probe drift reduction (bc_probe.cu): at most kProbeMaxCtas partial pairs of scratch.
+constexpr int kProbeMaxCtas = 1024;
+int probe_ctas();
+// Enqueue sum |cur - prev|, sum |prev| and their ratio into out[0..2] (device doubles),
+// using partials[0 .. 2 * max_parts) as scratch.  Two launches.
+int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, double *partials,
+                 int max_parts, double *out, void *stream, int64_t *launches);
 
 // Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst absolute).
 int launch_copy(const LayerEntry *layers, int n_layers, bc_dtype dtype, void *stream,

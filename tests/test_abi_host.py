@@ -220,3 +220,57 @@ def test_host_bf16_rounding_is_nearest_even():
     bits = synth.f32_to_bf16_bits(f)
     assert list(bits[:3]) == [0x3F80, 0x3F80, 0x3F82]
     np.testing.assert_array_equal(synth.bf16_bits_to_f32(bits)[3], np.float32(-2.5))
+
+
+# ------------------------------------------------------------------- sampler coefficients
+@pytest.mark.parametrize("alpha_t,alpha_bar_t", [(0.9999, 0.9999), (0.98, 0.5), (0.99, 1e-4),
+                                                  (1.0, 0.3)])
+def test_ddpm_coefficients_match_oracle(alpha_t, alpha_bar_t):
+    np.testing.assert_allclose(bc.bc_ddpm_coefficients(alpha_t, alpha_bar_t),
+                               oracle.ddpm_coefficients(alpha_t, alpha_bar_t), rtol=1e-14)
+
+
+@pytest.mark.parametrize("ab_t,ab_prev,eta", [(0.1, 0.2, 0.0), (0.1, 0.2, 1.0), (0.5, 0.9, 0.5),
+                                              (0.999, 1.0, 0.0), (1e-3, 0.05, 0.3)])
+def test_ddim_coefficients_match_oracle(ab_t, ab_prev, eta):
+    np.testing.assert_allclose(bc.bc_ddim_coefficients(ab_t, ab_prev, eta),
+                               oracle.ddim_coefficients(ab_t, ab_prev, eta), rtol=1e-13,
+                               atol=1e-15)
+
+
+def test_sampler_coefficient_errors():
+    for args in [(0.0, 0.5), (0.9, 1.0)]:
+        with pytest.raises(bc.BaryCacheError):
+            bc.bc_ddpm_coefficients(*args)
+    for args in [(0.5, 0.4, 0.0), (0.5, 0.6, -1.0), (0.1, 0.9, 5.0)]:
+        with pytest.raises(bc.BaryCacheError):
+            bc.bc_ddim_coefficients(*args)
+
+
+# ------------------------------------------------------------------- schedules
+def test_equal_schedule_matches_the_flops_tables_and_configs():
+    for interval, full in [(4, 14), (5, 11), (6, 10)]:      # Tables 1 and 3, H = 2
+        assert sum(bc.bc_schedule_equal(50, interval, 2)) == full
+    for name in ("c2i-512", "t2i-1024", "mmdit-t2i", "t2v"):
+        w = WORKLOADS[name]
+        assert bc.bc_schedule_equal(w.steps, w.interval, w.K) == \
+            [int(w.is_full(i)) for i in range(w.steps)]
+    assert bc.bc_schedule_equal(0, 3, 2) == []
+    with pytest.raises(bc.BaryCacheError):
+        bc.bc_schedule_equal(10, 0, 2)
+
+
+def test_adaptive_schedule_accumulates_and_resets():
+    st = bc.bc_adaptive_init(0.25, 2)
+    drifts = [0.0, 0.3, 0.1, 0.1, 0.06, 0.2, 0.01, 0.5, 0.0]
+    # steps 0, 1: window fills (full); then 0.1, 0.2 (skip), 0.26 >= 0.25 (full, reset),
+    # 0.2 (skip), 0.21 (skip), 0.71 (full, reset), 0.0 (skip)
+    want = [1, 1, 0, 0, 1, 0, 0, 1, 0]
+    assert [bc.bc_adaptive_decide(st, d) for d in drifts] == want
+    assert st.full_steps == 4 and st.steps == 9 and st.accumulated == 0.0
+    st0 = bc.bc_adaptive_init(0.0, 0)              # threshold 0: every step is full
+    assert all(bc.bc_adaptive_decide(st0, 0.0) for _ in range(5))
+    with pytest.raises(bc.BaryCacheError):
+        bc.bc_adaptive_decide(st, float("nan"))
+    with pytest.raises(bc.BaryCacheError):
+        bc.bc_adaptive_init(-1.0, 2)
