@@ -270,6 +270,26 @@ bc_status bc_adaptive_decide(bc_adaptive *s, double drift, int *run_full);
 bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
                          bc_dtype dtype, double *out, void *stream);
 
+/* The probe drift of bc_probe_drift without a handle and without any device allocation, for
+ * callers that cannot call cudaMalloc or let a library do so on their behalf: code running
+ * inside a host framework that owns every device allocation (a serving engine's memory
+ * planner, a plugin interface that forbids allocating outside it), or a latency-bound loop
+ * that cannot afford the implicit device synchronisation of cudaMalloc/cudaFree.  The paper
+ * has no counterpart; it is a deployment variant of bc_probe_drift.
+ * The reduction scratch is a 256 KiB array in the library's own device memory, which every
+ * device that loads the library holds until the process exits.  Its capacity bounds the
+ * input: n may be at most 1 GiB per tensor (2^29 bf16 or 2^28 fp32 elements); larger n is
+ * rejected with INVALID_ARG before anything is enqueued.  cur, prev: device, n elements of
+ * dtype, 16-byte aligned; out: 3 device doubles, as bc_probe_drift (same sums, within
+ * rounding: the partial sums are grouped differently).  The first call on a device looks up
+ * the array's device address (cudaGetSymbolAddress, with that device current); make that
+ * first call before any stream capture.  Every call shares the one array; it keeps the last
+ * call's partial sums, none of which a later call reads before rewriting them, so nothing
+ * needs clearing, but calls that overlap on the device (on different streams, or from
+ * different threads) race.  Errors: INVALID_ARG, ALIGNMENT, CUDA. */
+bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
+                                 double *out, void *stream);
+
 /* Counters of this handle (see bc_stats). */
 bc_status bc_cache_stats(bc_handle h, bc_stats *out);
 

@@ -102,6 +102,8 @@ _SIGNATURES = {
                            ctypes.c_int),
     "bc_probe_drift": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                         ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p], ctypes.c_int),
+    "bc_probe_drift_noalloc": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int,
+                                ctypes.c_void_p, ctypes.c_void_p], ctypes.c_int),
 }
 
 
@@ -319,3 +321,10 @@ def bc_probe_drift(h: int, cur: int, prev: int, n: int, dtype: int, out: int,
                    stream: int = 0) -> None:
     _check(lib().bc_probe_drift(h, cur or None, prev or None, n, dtype, out or None,
                                 stream or None), "bc_probe_drift")
+
+
+def bc_probe_drift_noalloc(cur: int, prev: int, n: int, dtype: int, out: int,
+                           stream: int = 0) -> None:
+    """bc_probe_drift without a handle or any device allocation (static library scratch)."""
+    _check(lib().bc_probe_drift_noalloc(cur or None, prev or None, n, dtype, out or None,
+                                        stream or None), "bc_probe_drift_noalloc")

@@ -853,6 +853,26 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
     return BC_OK;
 }
 
+bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
+                                 double *out, void *stream) {
+    t_last_error.clear();
+    if (!out || n < 0 || (n > 0 && (!cur || !prev)))
+        return fail(BC_ERR_INVALID_ARG, "need device cur, prev (n elements) and out[3]");
+    if (!dtype_valid(dtype)) return fail(BC_ERR_INVALID_ARG, "unknown dtype");
+    const int64_t max_n = bc::static_drift_max_elems(dtype);
+    if (n > max_n)
+        return fail(BC_ERR_INVALID_ARG,
+                    "n = %lld exceeds the no-allocation maximum of %lld elements (1 GiB per "
+                    "tensor); use bc_probe_drift with a cache handle",
+                    static_cast<long long>(n), static_cast<long long>(max_n));
+    if (!aligned16(cur) || !aligned16(prev))
+        return fail(BC_ERR_ALIGNMENT, "probe tensors must be 16-byte aligned");
+    int64_t launches = 0;
+    const int err = bc::launch_drift_static(cur, prev, n, dtype, out, stream, &launches);
+    if (err != cudaSuccess) return cuda_fail(err, "no-allocation drift");
+    return BC_OK;
+}
+
 bc_status bc_cache_stats(bc_handle h, bc_stats *out) {
     t_last_error.clear();
     bc_status s = check_handle(h);

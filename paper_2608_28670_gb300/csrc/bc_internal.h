@@ -105,6 +105,18 @@ int probe_ctas();
 int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, double *partials,
                  int max_parts, double *out, void *stream, int64_t *launches);
 
+// The no-allocation drift (bc_probe.cu): scratch is a file-scope device array of
+// kStaticDriftMaxTiles partial pairs (256 KiB), one pair per tile of
+// kStaticDriftTileGroups x 256 sixteen-byte groups of the input.
+constexpr int64_t kStaticDriftMaxTiles = 16384;
+constexpr int kStaticDriftTileGroups = 16;
+// Largest probe (elements of dtype) the static scratch can reduce: 1 GiB per tensor.
+int64_t static_drift_max_elems(bc_dtype dtype);
+// Enqueue the same sums as launch_drift using the static scratch; the first call on a
+// device looks up the array's address.  Two launches; *launches incremented per launch.
+int launch_drift_static(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
+                        double *out, void *stream, int64_t *launches);
+
 // Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst absolute).
 int launch_copy(const LayerEntry *layers, int n_layers, bc_dtype dtype, void *stream,
                 int64_t *launches);

@@ -14,6 +14,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <mutex>
 
 #include "bc_internal.h"
 
@@ -142,6 +143,124 @@ int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, d
     int err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     drift_final<<<1, kProbeThreads, 0, s>>>(partials, grid, out);
+    ++*launches;
+    return cudaGetLastError();
+}
+
+}  // namespace bc
+
+// ---------------------------------------------------------------------------------------
+// No-allocation variant (bc_probe_drift_noalloc).
+//
+// For callers that must not allocate device memory themselves nor have the library do it
+// for them, the scratch of the reduction lives in a file-scope device array that exists
+// for as long as the library is loaded, on every device that loads it.  Unlike the handle
+// variant above (one partial per CTA of a device-sized grid), this variant writes one
+// partial pair per fixed tile of the input, so its scratch need grows with the input and
+// is bounded by the array: kStaticDriftMaxTiles tiles of kStaticDriftTileGroups x 256
+// sixteen-byte groups, i.e. 1 GiB per probe tensor.  Every partial the final pass reads is
+// written earlier in the same call, so nothing needs clearing between calls; calls that
+// overlap on the device share the array and race.
+static __device__ __align__(256) double g_drift_scratch[2 * bc::kStaticDriftMaxTiles];
+
+namespace bc {
+namespace {
+
+__global__ void __launch_bounds__(kProbeThreads)
+    drift_tile_partials(const char *cur, const char *prev, int64_t n, int bf16, int64_t ntiles,
+                        double *partials) {
+    __shared__ double sh[kProbeThreads];
+    const int ev = bf16 ? 8 : 4;
+    const int64_t nvec = n / ev;
+    const int rem = static_cast<int>(n - nvec * ev);
+    constexpr int64_t kTileGroups = static_cast<int64_t>(kStaticDriftTileGroups) * kProbeThreads;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        double sd = 0.0, sp = 0.0;
+        for (int u = 0; u < kStaticDriftTileGroups; ++u) {
+            const int64_t g = tile * kTileGroups + static_cast<int64_t>(u) * kProbeThreads + threadIdx.x;
+            if (g < nvec) {
+                float c[8], p[8];
+                unpack(ld_nc16(cur + g * 16), c, bf16);
+                unpack(ld_nc16(prev + g * 16), p, bf16);
+                float gd = 0.0f, gp = 0.0f;
+                for (int e = 0; e < ev; ++e) {
+                    gd += fabsf(c[e] - p[e]);
+                    gp += fabsf(p[e]);
+                }
+                sd += gd;
+                sp += gp;
+            } else if (g == nvec && rem > 0) {  // the ragged last group, element by element
+                float gd = 0.0f, gp = 0.0f;
+                for (int e = 0; e < rem; ++e) {
+                    const float c = load1(cur, nvec * ev + e, bf16);
+                    const float p = load1(prev, nvec * ev + e, bf16);
+                    gd += fabsf(c - p);
+                    gp += fabsf(p);
+                }
+                sd += gd;
+                sp += gp;
+            }
+        }
+        sd = block_sum(sd, sh);
+        sp = block_sum(sp, sh);
+        if (threadIdx.x == 0) {
+            partials[2 * tile] = sd;
+            partials[2 * tile + 1] = sp;
+        }
+    }
+}
+
+std::mutex g_static_mu;
+constexpr int kMaxDevices = 64;
+double *g_static_scratch[kMaxDevices] = {};
+
+// Device address of g_drift_scratch on the current device.  In host code the array's name
+// only stands in for the symbol, so the address is looked up with cudaGetSymbolAddress,
+// once per device, with that device current (the first no-allocation call on it).
+int static_scratch(double **out) {
+    int dev = 0;
+    int err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_static_mu);
+    if (!g_static_scratch[dev]) {
+        void *p = nullptr;
+        err = cudaGetSymbolAddress(&p, g_drift_scratch);
+        if (err != cudaSuccess) return err;
+        g_static_scratch[dev] = static_cast<double *>(p);
+    }
+    *out = g_static_scratch[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
+
+int64_t static_drift_max_elems(bc_dtype dtype) {
+    const int64_t ev = dtype == BC_DTYPE_BF16 ? 8 : 4;
+    return kStaticDriftMaxTiles * kStaticDriftTileGroups * kProbeThreads * ev;
+}
+
+int launch_drift_static(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
+                        double *out, void *stream, int64_t *launches) {
+    double *scratch = nullptr;
+    int err = static_scratch(&scratch);
+    if (err != cudaSuccess) return err;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t ev = dtype == BC_DTYPE_BF16 ? 8 : 4;
+    const int64_t groups = (n + ev - 1) / ev;
+    constexpr int64_t kTileGroups = static_cast<int64_t>(kStaticDriftTileGroups) * kProbeThreads;
+    int64_t ntiles = (groups + kTileGroups - 1) / kTileGroups;
+    if (ntiles < 1) ntiles = 1;
+    if (ntiles > kStaticDriftMaxTiles) return cudaErrorInvalidValue;  // the caller checks first
+    int64_t grid = probe_ctas();
+    if (grid > ntiles) grid = ntiles;
+    drift_tile_partials<<<static_cast<int>(grid), kProbeThreads, 0, s>>>(
+        static_cast<const char *>(cur), static_cast<const char *>(prev), n,
+        dtype == BC_DTYPE_BF16 ? 1 : 0, ntiles, scratch);
+    ++*launches;
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    drift_final<<<1, kProbeThreads, 0, s>>>(scratch, static_cast<int>(ntiles), out);
     ++*launches;
     return cudaGetLastError();
 }
