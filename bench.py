@@ -11,7 +11,7 @@ Prints one JSON line (rank 0).  Default workload: the video DiT (60 x [1, 118800
 K = 3; 131 GB of cache, 175 GB of HBM traffic per step).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload t2v|mmdit-t2i|t2i-1024|c2i-512|c2i-256] [--K 3] [--sweep]
+                    [--workload t2v|mmdit-t2i|t2i-1024|c2i-512|c2i-256] [--K 3] [--no-sweep]
 """
 from __future__ import annotations
 
@@ -41,7 +41,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="t2v")
     ap.add_argument("--K", type=int, default=None)
-    ap.add_argument("--sweep", action="store_true", help="also time every K of the workload")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip timing the workload's other history depths K")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-e2e", action="store_true")
@@ -137,6 +138,22 @@ class ClockSampler:
                 "power_w_max": max(r[2] for r in rows)}
 
 
+# ----------------------------------------------------------------------------- ranks
+def max_over_ranks(value: float, dist=None, device="cuda") -> float:
+    """The slowest rank's value (time-like): all_reduce MAX, or the value itself at N = 1."""
+    if dist is None:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(bytes_per_rank: float, max_ms: float, world: int) -> float:
+    """Whole-job GB/s of N replicas that each move `bytes_per_rank` in at most `max_ms`."""
+    return bytes_per_rank * world / (max_ms * 1e-3) / 1e9
+
+
 # ----------------------------------------------------------------------------- GPU arm
 def window_targets(w, K):
     rep = w.representative(K)
@@ -203,13 +220,9 @@ def run_ours(args):
         clocks = ClockSampler(not args.no_clocks)
         total_ms, per_step, launches = time_forecast(run, args.steps, args.warmup, stream, dist)
         clk = clocks.stop()
-        ms = total_ms / args.steps
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = max_over_ranks(total_ms / args.steps, dist)
         alg = run.algorithmic_bytes()
-        value = alg * world / (ms * 1e-3) / 1e9
+        value = job_throughput(alg, ms, world)
         elems = run.w.layer_numel * run.n_feat + (run.numels[-1] if run.euler else 0)
         launches_per_step = launches / args.steps
         kernel_ms = statistics.mean(per_step) / max(launches_per_step, 1)
@@ -257,7 +270,7 @@ def run_ours(args):
         }
         if clk:
             result["clocks"] = clk
-        if args.sweep and w.K_sweep:
+        if not args.no_sweep and w.K_sweep:
             sweep = {}
             run.close()
             run = None
@@ -277,10 +290,10 @@ def run_ours(args):
                     torch.cuda.empty_cache()
             result["sweep"] = sweep
             run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
+        if not args.no_e2e:      # before the CPU leg, which loads the host memory system
+            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
             result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
-        if not args.no_e2e:
-            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
         if not args.no_extra:
             result["push"] = time_push(run, args.steps)
     finally:
@@ -478,13 +491,9 @@ def e2e(run, steps, world, dist, chunk_layers=6):
         b.record()
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
-        ms = a.elapsed_time(b) / steps
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = max_over_ranks(a.elapsed_time(b) / steps, dist)
         alg = run.algorithmic_bytes()
-        return {"value": round(alg * world / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+        return {"value": round(job_throughput(alg, ms, world), 1), "unit": "GB/s",
                 "h2d_bytes_per_step": total,
                 "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
                 "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
@@ -498,6 +507,68 @@ def e2e(run, steps, world, dist, chunk_layers=6):
 
 
 CHUNK = 1 << 22   # elements per oracle call in the CPU samples
+
+
+def _oracle_pool_init():
+    import oracle
+    oracle.build()
+    oracle._load()
+
+
+def _oracle_task(args):
+    """One oracle call on a chunk held in shared memory (runs in a spawned worker)."""
+    from multiprocessing import shared_memory
+    import numpy as np
+    import oracle
+    shm_name, dtype, m, total, off, size, W = args
+    shm = shared_memory.SharedMemory(name=shm_name)
+    try:
+        arr = np.ndarray((m, total), dtype=dtype, buffer=shm.buf)
+        F = [arr[j, off:off + size] for j in range(m)]
+        oracle.combine(F, W)
+        del F, arr
+    finally:
+        shm.close()
+    return size
+
+
+class OraclePool:
+    """The unmodified fp64 oracle on every host core: a spawn pool of one worker per core,
+    each running oracle.combine on chunks of a sample held in shared memory."""
+
+    def __init__(self, sample: list, W, workers: int | None = None):
+        import multiprocessing as mp
+        from multiprocessing import shared_memory
+        import numpy as np
+        self.m = len(sample)
+        self.dtype = sample[0].dtype
+        self.total = sample[0].size
+        self.shm = shared_memory.SharedMemory(create=True,
+                                              size=self.m * self.total * sample[0].itemsize)
+        arr = np.ndarray((self.m, self.total), dtype=self.dtype, buffer=self.shm.buf)
+        for j in range(self.m):
+            arr[j] = sample[j]
+        del arr
+        self.W = [float(w) for w in W]
+        self.workers = workers or os.cpu_count() or 1
+        self.pool = mp.get_context("spawn").Pool(self.workers, initializer=_oracle_pool_init)
+        self.tasks = [(self.shm.name, self.dtype, self.m, self.total, off,
+                       min(CHUNK, self.total - off), self.W)
+                      for off in range(0, self.total, CHUNK)]
+        self.pool.map(_oracle_task, self.tasks[:self.workers])        # warm the workers
+
+    def run(self, passes: int = 1):
+        """Process the whole sample `passes` times; returns (elements, seconds)."""
+        t0 = time.perf_counter()
+        done = sum(sum(self.pool.map(_oracle_task, self.tasks, chunksize=1))
+                   for _ in range(passes))
+        return done, time.perf_counter() - t0
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+        self.shm.close()
+        self.shm.unlink()
 
 
 def _time_oracle(chunks, W, seconds):
@@ -516,9 +587,11 @@ def _time_oracle(chunks, W, seconds):
 
 
 def cpu_baseline_from_device(run, seconds):
-    """The fp64 oracle, single-threaded on the host, over a bounded sample of the same
-    workload: chunks of 4 Mi elements of the live history slots (copied to the host first,
-    outside the timed region), layers round-robin."""
+    """The fp64 oracle on the host over a bounded sample of the same workload: 64 chunks of
+    4 Mi consecutive elements of the live history slots (copied to the host first, outside
+    the timed region; layers round-robin; 1.5 GB of bf16, far beyond the host caches).  Timed
+    on every host core (spawned workers running the unmodified oracle) and, for reference, on
+    one core."""
     import numpy as np
     import oracle
     from paper_2608_28670_gb300.runner import device_view
@@ -527,31 +600,39 @@ def cpu_baseline_from_device(run, seconds):
     W = oracle.paper_weights(list(p.nodes), p.t)
     m = len(p.nodes)
     slots = [bc_slot_ptrs(run, j) for j in range(m)]
-
-    def chunk(c):
+    n_chunks = 64
+    parts = [[] for _ in range(m)]
+    for c in range(n_chunks):
         l = c % run.n_feat
         n = run.numels[l]
         size = min(CHUNK, n)
         off = ((c * 2654435761) % max(1, n - size + 1)) // 8 * 8
-        F = []
         for j in range(m):
             v = device_view(slots[j][l], n, run.w.dtype)[off:off + size].cpu().numpy()
-            F.append(v.view(np.uint16) if v.dtype == np.int16 else v)
-        return F
-
-    first = chunk(0)
-    n1, t1 = _time_oracle([first], W, 1e9)
-    want = max(1, min(400, int(seconds / max(t1, 1e-6))))
-    chunks = [chunk(c) for c in range(1, want)]
-    n2, t2 = _time_oracle(chunks, W, seconds)
-    elems, secs = n1 + n2, t1 + t2
+            parts[j].append(v.view(np.uint16) if v.dtype == np.int16 else v)
+    sample = [np.concatenate(parts[j]) for j in range(m)]
     per_elem = run.algorithmic_bytes() / (run.w.layer_numel * run.n_feat)
-    return {"value": round(elems * per_elem / secs / 1e9, 4), "unit": "GB/s", "cores": 1,
-            "kind": "oracle",
-            "elems_per_s": round(elems / secs, 1),
-            "sample": f"{elems} elements ({len(chunks) + 1} chunks of <= {CHUNK} consecutive "
-                      f"elements, layers round-robin) of the K={m} history slots, fp64 oracle, "
-                      f"{secs:.1f} s"}
+
+    # one core
+    one = [[sample[j][o:o + CHUNK] for j in range(m)] for o in range(0, sample[0].size, CHUNK)]
+    n1, t1 = _time_oracle(one, W, seconds / 3)
+    # every core
+    pool = OraclePool(sample, W)
+    try:
+        e0, s0 = pool.run(1)
+        passes = max(1, int((2 * seconds / 3) / max(s0, 1e-3)))
+        e1, s1 = pool.run(passes)
+        elems, secs = e0 + e1, s0 + s1
+        cores = pool.workers
+    finally:
+        pool.close()
+    return {"value": round(elems * per_elem / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
+            "kind": "oracle", "elems_per_s": round(elems / secs, 1),
+            "sample": f"{sample[0].size} elements (64 chunks of {CHUNK} consecutive elements, "
+                      f"layers round-robin) of the K={m} history slots, processed {1 + passes} "
+                      f"times by {cores} spawned workers running the fp64 oracle, {secs:.1f} s",
+            "single_core": {"value": round(n1 * per_elem / t1 / 1e9, 4), "cores": 1,
+                            "elems_per_s": round(n1 / t1, 1), "seconds": round(t1, 1)}}
 
 
 def bc_slot_ptrs(run, j):
@@ -573,7 +654,7 @@ def run_reference(args):
     w = WORKLOADS[args.workload]
     K = args.K or w.K
     p = w.representative(K)
-    n = 1 << 25                       # 32 Mi elements per node: inputs larger than the host L3
+    n = 1 << 25                       # 32 Mi elements per node: inputs beyond the host L3
     nodes_oldest_first = list(reversed(p.nodes))
     feats = synth.host_trajectories([(n,)], [w.tau(t) for t in nodes_oldest_first],
                                     dtype="bf16" if w.elem_bytes == 2 else "f32",
@@ -581,26 +662,28 @@ def run_reference(args):
     F = [f[0] for f in reversed(feats)]        # newest first
     W = oracle.paper_weights(list(p.nodes), p.t)
     per_elem = (K * w.elem_bytes + w.elem_bytes)
-    reps = 1
-    for _ in range(args.warmup):
-        for _ in range(reps):
-            oracle.combine(F, W)
-    times = []
-    for _ in range(args.steps):
-        t0 = time.perf_counter()
-        for _ in range(reps):
-            oracle.combine(F, W)
-        times.append(time.perf_counter() - t0)
+    pool = OraclePool(F, W)
+    try:
+        for _ in range(args.warmup):
+            pool.run(1)
+        times = []
+        for _ in range(args.steps):
+            _, secs = pool.run(1)
+            times.append(secs)
+        cores = pool.workers
+    finally:
+        pool.close()
     ms = 1e3 * sum(times) / len(times)
-    value = reps * n * per_elem / (ms * 1e-3) / 1e9
-    sample = f"{reps} x {n} elements per step of one [{n}] bf16 slice at K={K}, fp64 oracle"
+    value = n * per_elem / (ms * 1e-3) / 1e9
+    sample = (f"{n} elements per step of one [{n}] slice at K={K} (host-generated with the "
+              f"workload's recipe), fp64 oracle on {cores} spawned workers")
     out = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": w.name, "K": K, "nodes": list(p.nodes), "target": p.t,
-                      "sample_elements_per_step": reps * n},
-           "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1,
+                      "sample_elements_per_step": n},
+           "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores,
                             "kind": "oracle", "sample": sample},
            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}

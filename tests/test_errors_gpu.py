@@ -1,0 +1,117 @@
+"""Failure behaviour of the C ABI on a GPU: every fault is injected on the host side (bad
+arguments, wrong call order, a device allocation the GPU cannot satisfy) and must come back
+as a status code with a message, leaving the context usable."""
+import pytest
+import torch
+
+from paper_2608_28670_gb300 import barycache as bc
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build_libraries()
+    torch.cuda.set_device(0)
+
+
+def _status(fn, *args):
+    with pytest.raises(bc.BaryCacheError) as ei:
+        fn(*args)
+    assert bc.lib().bc_last_error().decode()
+    return ei.value.status
+
+
+def s():
+    return torch.cuda.current_stream().cuda_stream
+
+
+def test_forecast_before_any_push_is_not_ready():
+    h = bc.bc_cache_create([1024], 3, bc.DTYPE_BF16)
+    try:
+        out = torch.empty(1024, dtype=torch.bfloat16, device="cuda")
+        assert _status(bc.bc_forecast, h, 0.5, [out.data_ptr()], bc.DTYPE_BF16, s()) == \
+            bc.ERR_NOT_READY
+        assert _status(bc.bc_coefficients, h, 0.5) == bc.ERR_NOT_READY
+        assert _status(bc.bc_forecast_flat, h, 0.5, out.data_ptr(), s()) == bc.ERR_NOT_READY
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_duplicate_nodes_and_ring_eviction():
+    h = bc.bc_cache_create([256], 2, bc.DTYPE_F32)
+    try:
+        x = torch.zeros(256, device="cuda")
+        bc.bc_cache_push(h, [x.data_ptr()], 0.9, s())
+        assert _status(bc.bc_cache_push, h, [x.data_ptr()], 0.9, s()) == bc.ERR_DUPLICATE_NODE
+        bc.bc_cache_push(h, [x.data_ptr()], 0.8, s())
+        # window full (0.8, 0.9): pushing 0.9 again evicts 0.9 first, so it is not a duplicate
+        bc.bc_cache_push(h, [x.data_ptr()], 0.9, s())
+        assert bc.bc_cache_nodes(h) == [0.9, 0.8]
+        # 0.8 is the oldest and would be evicted by this commit: allowed; 0.9 stays: duplicate
+        assert _status(bc.bc_cache_commit, h, 0.9) == bc.ERR_DUPLICATE_NODE
+        assert _status(bc.bc_cache_commit, h, float("nan")) == bc.ERR_INVALID_ARG
+        bc.bc_cache_reset(h)
+        assert bc.bc_cache_nodes(h) == []
+        assert bc.bc_cache_stats(h)["pushes"] == 3
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_pointer_checks():
+    h = bc.bc_cache_create([4096, 100], 2, bc.DTYPE_BF16)
+    try:
+        x = torch.zeros(8192, dtype=torch.bfloat16, device="cuda")
+        p = x.data_ptr()
+        assert _status(bc.bc_cache_push, h, [p + 2, p], 0.5, s()) == bc.ERR_ALIGNMENT
+        assert _status(bc.bc_cache_push, h, [p, 0], 0.5, s()) == bc.ERR_INVALID_ARG
+        slot = bc.bc_cache_next_slot_ptrs(h, 2)
+        assert _status(bc.bc_cache_push, h, [slot[0], p], 0.5, s()) == bc.ERR_INVALID_ARG
+        bc.bc_cache_push(h, [p, p], 0.5, s())
+        assert _status(bc.bc_forecast, h, 0.4, [p + 16 + 2, None], bc.DTYPE_BF16, s()) == \
+            bc.ERR_ALIGNMENT
+        live = bc.bc_cache_slot_ptrs(h, 0, 2)
+        assert _status(bc.bc_forecast, h, 0.4, [live[0], None], bc.DTYPE_BF16, s()) == \
+            bc.ERR_INVALID_ARG                                   # output inside the arena
+        assert _status(bc.bc_forecast, h, 0.4, [p, None], 7, s()) == bc.ERR_INVALID_ARG
+        assert _status(bc.bc_forecast_step, h, 0.4, -0.1, [p, None], bc.DTYPE_BF16, 0, p,
+                       bc.DTYPE_F32, s()) == bc.ERR_INVALID_ARG       # output aliases x
+        assert _status(bc.bc_forecast_step, h, 0.4, -0.1, [None, None], bc.DTYPE_BF16, 5, p,
+                       bc.DTYPE_F32, s()) == bc.ERR_INVALID_ARG       # no such layer
+        assert _status(bc.bc_forecast, h, float("inf"), [p, None], bc.DTYPE_BF16, s()) == \
+            bc.ERR_INVALID_ARG
+        assert _status(bc.bc_cache_slot_ptrs, h, 1, 2) == bc.ERR_INVALID_ARG
+    finally:
+        bc.bc_cache_destroy(h)
+    torch.cuda.synchronize()                     # the context is still usable
+
+
+def test_destroyed_handle_is_rejected():
+    h = bc.bc_cache_create([64], 2, bc.DTYPE_F32)
+    bc.bc_cache_destroy(h)
+    assert _status(bc.bc_cache_bytes, h) == bc.ERR_BAD_HANDLE
+    assert _status(bc.bc_cache_destroy, h) == bc.ERR_BAD_HANDLE
+    assert _status(bc.bc_forecast, h, 0.1, [None], bc.DTYPE_F32, s()) == bc.ERR_BAD_HANDLE
+
+
+def test_device_out_of_memory_is_a_status():
+    free, total = torch.cuda.mem_get_info()
+    numel = (total // 2) * 2                     # K = 2 slots of `total` bytes of bf16 each
+    assert _status(bc.bc_cache_create, [numel // 2], 2, bc.DTYPE_BF16) in (bc.ERR_OOM,)
+    h = bc.bc_cache_create([1024], 2, bc.DTYPE_BF16)   # the device still allocates afterwards
+    bc.bc_cache_destroy(h)
+
+
+def test_degenerate_weights_status():
+    h = bc.bc_cache_create([64], 2, bc.DTYPE_F32,
+                           bc.make_params(mode=bc.MODE_PAPER, delta=1.0, eta=0.0))
+    try:
+        x = torch.zeros(64, device="cuda")
+        bc.bc_cache_push(h, [x.data_ptr()], 0.02, s())
+        bc.bc_cache_push(h, [x.data_ptr()], 0.01, s())
+        out = torch.empty(64, device="cuda")
+        assert _status(bc.bc_forecast, h, 0.0, [out.data_ptr()], bc.DTYPE_F32, s()) == \
+            bc.ERR_DEGENERATE_WEIGHTS
+    finally:
+        bc.bc_cache_destroy(h)
