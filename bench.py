@@ -295,6 +295,7 @@ def run_ours(args):
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
             result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
         if not args.no_extra:
+            result["probe_drift"] = time_probe(run, args.steps)
             result["push"] = time_push(run, args.steps)
     finally:
         if run is not None:
@@ -345,6 +346,34 @@ def time_push(run, steps):
     return {"GB/s": round(2 * slot / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
             "bytes_per_push": 2 * slot, "pushes": steps,
             "what": "grouped byte-exact copy of one slot (read + write)"}
+
+
+def time_probe(run, steps):
+    """Row f3: the probe drift of the adaptive schedule over one cached layer (newest vs the
+    previous node's copy of layer 0): 2 x numel x b bytes, two launches per call."""
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    if len(run.problem.nodes) < 2:
+        return None
+    n = run.numels[0]
+    cur = bc.bc_cache_slot_ptrs(run.h, 0, len(run.numels))[0]
+    prev = bc.bc_cache_slot_ptrs(run.h, 1, len(run.numels))[0]
+    out = torch.empty(3, dtype=torch.float64, device="cuda")
+    for _ in range(3):
+        bc.bc_probe_drift(run.h, cur, prev, n, run.w.dtype, out.data_ptr(), run.stream)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(steps):
+        bc.bc_probe_drift(run.h, cur, prev, n, run.w.dtype, out.data_ptr(), run.stream)
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    nbytes = 2 * n * run.w.elem_bytes
+    return {"GB/s": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
+            "elements": n, "bytes_per_call": nbytes, "drift": round(float(out[2].item()), 6),
+            "what": "bc_probe_drift over layer 0 (newest vs previous node)"}
 
 
 def time_fused(args, stream, dist):

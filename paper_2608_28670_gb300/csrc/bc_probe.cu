@@ -5,9 +5,11 @@
 //     drift = sum_e |cur[e] - prev[e]| / sum_e |prev[e]|
 //
 // Two launches with a fixed reduction order, so the result is bitwise reproducible for a
-// given device: (1) a persistent grid streams both tensors once in 16-byte groups, each
-// thread sums a group in fp32 and accumulates the group sums in fp64 (fp64 per element
-// would outrun GB300's fp64 rate), and every CTA writes its two partial sums to scratch;
+// given device: (1) a persistent grid streams both tensors once in 16-byte groups (four
+// groups of loads in flight per thread), each thread sums a group in fp32 and accumulates
+// the group sums with compensated (Kahan) fp32 addition, so the error stays near two fp32
+// ulps however long the stream is, without touching GB300's slow fp64 pipe per element;
+// every CTA adds its threads' sums in fp64 and writes its two partial sums to scratch;
 // (2) one CTA adds the partials in index order and writes {sum |d|, sum |prev|, ratio}.
 // HBM-bound: 2 * n * sizeof(T) bytes.  No atomics, no waits.
 #include <cuda_bf16.h>
@@ -31,8 +33,9 @@ __device__ __forceinline__ uint4 ld_nc16(const void *p) {
     return r;
 }
 
-__device__ __forceinline__ void unpack(uint4 r, float *f, bool bf16) {
-    if (bf16) {
+template <bool kBf16>
+__device__ __forceinline__ void unpack(uint4 r, float *f) {
+    if constexpr (kBf16) {
         const uint32_t w[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -45,10 +48,45 @@ __device__ __forceinline__ void unpack(uint4 r, float *f, bool bf16) {
     }
 }
 
-__device__ __forceinline__ float load1(const char *p, int64_t e, bool bf16) {
-    if (bf16) return __uint_as_float(static_cast<uint32_t>(reinterpret_cast<const uint16_t *>(p)[e]) << 16);
+template <bool kBf16>
+__device__ __forceinline__ float load1(const char *p, int64_t e) {
+    if constexpr (kBf16)
+        return __uint_as_float(static_cast<uint32_t>(reinterpret_cast<const uint16_t *>(p)[e]) << 16);
     return reinterpret_cast<const float *>(p)[e];
 }
+
+// Compensated fp32 accumulator (Kahan): the rounding error of every addition is carried
+// into the next, so a long sum keeps about fp32 precision.  Inputs are sums of |x| >= 0.
+struct Kahan {
+    float s = 0.0f, c = 0.0f;
+    __device__ __forceinline__ void add(float x) {
+        const float y = x - c;
+        const float t = s + y;
+        c = (t - s) - y;
+        s = t;
+    }
+    __device__ __forceinline__ double value() const {
+        return static_cast<double>(s) - static_cast<double>(c);
+    }
+};
+
+// Sum |c - p| and |p| over one 16-byte group of each tensor (fp32, fixed order).
+template <bool kBf16>
+__device__ __forceinline__ void group_sums(uint4 rc, uint4 rp, float &gd, float &gp) {
+    constexpr int ev = kBf16 ? 8 : 4;
+    float c[8], p[8];
+    unpack<kBf16>(rc, c);
+    unpack<kBf16>(rp, p);
+    gd = 0.0f;
+    gp = 0.0f;
+#pragma unroll
+    for (int e = 0; e < ev; ++e) {
+        gd += fabsf(c[e] - p[e]);
+        gp += fabsf(p[e]);
+    }
+}
+
+constexpr int kGroupsInFlight = 4;
 
 // Fixed-order tree sum of one double per thread over the CTA (kProbeThreads threads).
 __device__ __forceinline__ double block_sum(double v, double *sh) {
@@ -63,39 +101,50 @@ __device__ __forceinline__ double block_sum(double v, double *sh) {
     return r;
 }
 
+template <bool kBf16>
 __global__ void __launch_bounds__(kProbeThreads)
-    drift_partials(const char *cur, const char *prev, int64_t n, int bf16, double *partials) {
+    drift_partials(const char *cur, const char *prev, int64_t n, double *partials) {
     __shared__ double sh[kProbeThreads];
-    const int ev = bf16 ? 8 : 4;
+    constexpr int ev = kBf16 ? 8 : 4;
     const int64_t nvec = n / ev;
-    double sd = 0.0, sp = 0.0;
-    const int64_t stride = static_cast<int64_t>(gridDim.x) * kProbeThreads;
-    for (int64_t v = static_cast<int64_t>(blockIdx.x) * kProbeThreads + threadIdx.x; v < nvec;
-         v += stride) {
-        float c[8], p[8];
-        unpack(ld_nc16(cur + v * 16), c, bf16);
-        unpack(ld_nc16(prev + v * 16), p, bf16);
-        float gd = 0.0f, gp = 0.0f;
-        for (int e = 0; e < ev; ++e) {
-            gd += fabsf(c[e] - p[e]);
-            gp += fabsf(p[e]);
+    Kahan sd, sp;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * kProbeThreads * kGroupsInFlight;
+    for (int64_t base = static_cast<int64_t>(blockIdx.x) * kProbeThreads * kGroupsInFlight +
+                        threadIdx.x;
+         base < nvec; base += stride) {
+        uint4 rc[kGroupsInFlight], rp[kGroupsInFlight];
+#pragma unroll
+        for (int u = 0; u < kGroupsInFlight; ++u) {
+            const int64_t g = base + static_cast<int64_t>(u) * kProbeThreads;
+            if (g < nvec) {
+                rc[u] = ld_nc16(cur + g * 16);
+                rp[u] = ld_nc16(prev + g * 16);
+            }
         }
-        sd += gd;
-        sp += gp;
+#pragma unroll
+        for (int u = 0; u < kGroupsInFlight; ++u) {
+            const int64_t g = base + static_cast<int64_t>(u) * kProbeThreads;
+            if (g < nvec) {
+                float gd, gp;
+                group_sums<kBf16>(rc[u], rp[u], gd, gp);
+                sd.add(gd);
+                sp.add(gp);
+            }
+        }
     }
     if (blockIdx.x == 0) {  // ragged tail: fewer than one 16-byte group
         const int64_t e = nvec * ev + threadIdx.x;
         if (e < n) {
-            const float c = load1(cur, e, bf16), p = load1(prev, e, bf16);
-            sd += fabsf(c - p);
-            sp += fabsf(p);
+            const float c = load1<kBf16>(cur, e), p = load1<kBf16>(prev, e);
+            sd.add(fabsf(c - p));
+            sp.add(fabsf(p));
         }
     }
-    sd = block_sum(sd, sh);
-    sp = block_sum(sp, sh);
+    const double bd = block_sum(sd.value(), sh);
+    const double bp = block_sum(sp.value(), sh);
     if (threadIdx.x == 0) {
-        partials[2 * blockIdx.x] = sd;
-        partials[2 * blockIdx.x + 1] = sp;
+        partials[2 * blockIdx.x] = bd;
+        partials[2 * blockIdx.x + 1] = bp;
     }
 }
 
@@ -136,9 +185,12 @@ int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, d
     int grid = probe_ctas();
     if (grid > max_parts) grid = max_parts;
     if (want < grid) grid = static_cast<int>(want);
-    drift_partials<<<grid, kProbeThreads, 0, s>>>(static_cast<const char *>(cur),
-                                                  static_cast<const char *>(prev), n,
-                                                  dtype == BC_DTYPE_BF16 ? 1 : 0, partials);
+    if (dtype == BC_DTYPE_BF16)
+        drift_partials<true><<<grid, kProbeThreads, 0, s>>>(
+            static_cast<const char *>(cur), static_cast<const char *>(prev), n, partials);
+    else
+        drift_partials<false><<<grid, kProbeThreads, 0, s>>>(
+            static_cast<const char *>(cur), static_cast<const char *>(prev), n, partials);
     ++*launches;
     int err = cudaGetLastError();
     if (err != cudaSuccess) return err;
@@ -166,46 +218,56 @@ static __device__ __align__(256) double g_drift_scratch[2 * bc::kStaticDriftMaxT
 namespace bc {
 namespace {
 
+template <bool kBf16>
 __global__ void __launch_bounds__(kProbeThreads)
-    drift_tile_partials(const char *cur, const char *prev, int64_t n, int bf16, int64_t ntiles,
+    drift_tile_partials(const char *cur, const char *prev, int64_t n, int64_t ntiles,
                         double *partials) {
     __shared__ double sh[kProbeThreads];
-    const int ev = bf16 ? 8 : 4;
+    constexpr int ev = kBf16 ? 8 : 4;
     const int64_t nvec = n / ev;
     const int rem = static_cast<int>(n - nvec * ev);
     constexpr int64_t kTileGroups = static_cast<int64_t>(kStaticDriftTileGroups) * kProbeThreads;
+    static_assert(kStaticDriftTileGroups % kGroupsInFlight == 0, "whole rounds per tile");
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        double sd = 0.0, sp = 0.0;
-        for (int u = 0; u < kStaticDriftTileGroups; ++u) {
-            const int64_t g = tile * kTileGroups + static_cast<int64_t>(u) * kProbeThreads + threadIdx.x;
-            if (g < nvec) {
-                float c[8], p[8];
-                unpack(ld_nc16(cur + g * 16), c, bf16);
-                unpack(ld_nc16(prev + g * 16), p, bf16);
-                float gd = 0.0f, gp = 0.0f;
-                for (int e = 0; e < ev; ++e) {
-                    gd += fabsf(c[e] - p[e]);
-                    gp += fabsf(p[e]);
+        Kahan sd, sp;
+        for (int r = 0; r < kStaticDriftTileGroups; r += kGroupsInFlight) {
+            uint4 rc[kGroupsInFlight], rp[kGroupsInFlight];
+            const int64_t g0 = tile * kTileGroups + static_cast<int64_t>(r) * kProbeThreads +
+                               threadIdx.x;
+#pragma unroll
+            for (int u = 0; u < kGroupsInFlight; ++u) {
+                const int64_t g = g0 + static_cast<int64_t>(u) * kProbeThreads;
+                if (g < nvec) {
+                    rc[u] = ld_nc16(cur + g * 16);
+                    rp[u] = ld_nc16(prev + g * 16);
                 }
-                sd += gd;
-                sp += gp;
-            } else if (g == nvec && rem > 0) {  // the ragged last group, element by element
-                float gd = 0.0f, gp = 0.0f;
-                for (int e = 0; e < rem; ++e) {
-                    const float c = load1(cur, nvec * ev + e, bf16);
-                    const float p = load1(prev, nvec * ev + e, bf16);
-                    gd += fabsf(c - p);
-                    gp += fabsf(p);
+            }
+#pragma unroll
+            for (int u = 0; u < kGroupsInFlight; ++u) {
+                const int64_t g = g0 + static_cast<int64_t>(u) * kProbeThreads;
+                if (g < nvec) {
+                    float gd, gp;
+                    group_sums<kBf16>(rc[u], rp[u], gd, gp);
+                    sd.add(gd);
+                    sp.add(gp);
+                } else if (g == nvec && rem > 0) {  // the ragged last group, element by element
+                    float gd = 0.0f, gp = 0.0f;
+                    for (int e = 0; e < rem; ++e) {
+                        const float c = load1<kBf16>(cur, nvec * ev + e);
+                        const float p = load1<kBf16>(prev, nvec * ev + e);
+                        gd += fabsf(c - p);
+                        gp += fabsf(p);
+                    }
+                    sd.add(gd);
+                    sp.add(gp);
                 }
-                sd += gd;
-                sp += gp;
             }
         }
-        sd = block_sum(sd, sh);
-        sp = block_sum(sp, sh);
+        const double bd = block_sum(sd.value(), sh);
+        const double bp = block_sum(sp.value(), sh);
         if (threadIdx.x == 0) {
-            partials[2 * tile] = sd;
-            partials[2 * tile + 1] = sp;
+            partials[2 * tile] = bd;
+            partials[2 * tile + 1] = bp;
         }
     }
 }
@@ -254,9 +316,12 @@ int launch_drift_static(const void *cur, const void *prev, int64_t n, bc_dtype d
     if (ntiles > kStaticDriftMaxTiles) return cudaErrorInvalidValue;  // the caller checks first
     int64_t grid = probe_ctas();
     if (grid > ntiles) grid = ntiles;
-    drift_tile_partials<<<static_cast<int>(grid), kProbeThreads, 0, s>>>(
-        static_cast<const char *>(cur), static_cast<const char *>(prev), n,
-        dtype == BC_DTYPE_BF16 ? 1 : 0, ntiles, scratch);
+    if (dtype == BC_DTYPE_BF16)
+        drift_tile_partials<true><<<static_cast<int>(grid), kProbeThreads, 0, s>>>(
+            static_cast<const char *>(cur), static_cast<const char *>(prev), n, ntiles, scratch);
+    else
+        drift_tile_partials<false><<<static_cast<int>(grid), kProbeThreads, 0, s>>>(
+            static_cast<const char *>(cur), static_cast<const char *>(prev), n, ntiles, scratch);
     ++*launches;
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
