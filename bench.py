@@ -63,11 +63,18 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+KERNEL_CODE_END = "// ------------------------------------------------------------------ launch plumbing"
+
+
 def kernel_source_hash() -> str:
+    """Hash of the forecast kernel's device code (bc_forecast.cu up to its host launch
+    plumbing) and of the shared layout header: a change there voids a stored ncu figure."""
     h = hashlib.sha256()
-    for f in ("bc_forecast.cu", "bc_internal.h"):
-        with open(os.path.join(ROOT, "paper_2608_28670_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+    csrc = os.path.join(ROOT, "paper_2608_28670_gb300", "csrc")
+    with open(os.path.join(csrc, "bc_forecast.cu"), "rb") as fh:
+        h.update(fh.read().split(KERNEL_CODE_END.encode(), 1)[0])
+    with open(os.path.join(csrc, "bc_internal.h"), "rb") as fh:
+        h.update(fh.read())
     return h.hexdigest()[:16]
 
 

@@ -23,6 +23,11 @@
  * Everything is evaluated in double precision.  Stored inputs (fp32 or bf16) convert to
  * double exactly, so the oracle's result is the mathematically defined value up to fp64
  * rounding.
+ *
+ * Pins (tests/test_oracle_pins.py, tests/test_oracle_samplers.py): every function is checked
+ * against closed forms, identities or library routines.  For the paper's weights with a decay
+ * power delta != 1 the paper fixes no value: those are pinned by invariants and limits only
+ * (scale invariance, the delta -> 0 limit, sign alternation, unit sum, translation invariance).
  */
 #include <math.h>
 #include <stdint.h>

@@ -375,16 +375,22 @@ __global__ void __launch_bounds__(kThreads) copy_kernel(const __grid_constant__ 
 
 // ------------------------------------------------------------------ launch plumbing
 
-int g_sm_count = 0;
-
+// SM count of the current device, cached per device.
 int sm_count() {
-    if (g_sm_count == 0) {
-        int dev = 0, n = 0;
-        cudaGetDevice(&dev);
+    static int cached[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+    if (dev >= 64) {
+        int n = 0;
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        g_sm_count = n > 0 ? n : 1;
+        return n > 0 ? n : 1;
     }
-    return g_sm_count;
+    if (cached[dev] == 0) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cached[dev] = n > 0 ? n : 1;
+    }
+    return cached[dev];
 }
 
 // Resident CTAs per SM for a kernel, optionally capped (the forecast runs best at two

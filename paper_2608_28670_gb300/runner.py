@@ -9,13 +9,11 @@ over windows of layers (NULL outputs elsewhere), reusing one window of output bu
 """
 from __future__ import annotations
 
-from dataclasses import dataclass
-
 import torch
 
 from . import barycache as bc
 from . import synth
-from .configs import Workload, Problem
+from .configs import Workload
 
 SEED = 2026
 
@@ -30,15 +28,6 @@ def device_view(ptr: int, n: int, dtype: int) -> torch.Tensor:
     """Zero-copy 1-D torch view of `n` elements at device address `ptr` (bf16 as int16)."""
     typestr = "<f4" if dtype == bc.DTYPE_F32 else "<i2"
     return torch.as_tensor(_CudaArray(ptr, n, typestr), device="cuda")
-
-
-@dataclass
-class Plan:
-    K: int
-    problem: Problem
-    out_dtype: int
-    window: int          # layers per forecast call (n_layers = one call)
-    calls: int
 
 
 class WorkloadRun:
@@ -96,9 +85,6 @@ class WorkloadRun:
         synth.fill_device(self.x.data_ptr(), bc.DTYPE_F32, self.x.numel(), seed=self.seed + 1,
                           tensor_id=0, step_id=0, tau=0.0, degree=0, noise_std=0.0,
                           stream=self.stream)
-
-    def plan(self) -> Plan:
-        return Plan(self.K, self.problem, self.out_dtype, self.window, self.calls)
 
     # ------------------------------------------------------------------ the hot path
     def out_ptrs(self, call: int) -> list[int | None]:
