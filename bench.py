@@ -310,6 +310,11 @@ def run_ours(args):
     if not args.no_extra and w.name != "mmdit-t2i":
         torch.cuda.empty_cache()
         result["fused_step"] = time_fused(args, stream, dist)
+    if not args.no_extra:
+        torch.cuda.empty_cache()
+        result["sampling_loop"] = time_sampling_loop(stream)
+        torch.cuda.empty_cache()
+        result["blockwise"] = time_blockwise(stream, args.steps)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -381,6 +386,118 @@ def time_probe(run, steps):
     return {"GB/s": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
             "elements": n, "bytes_per_call": nbytes, "drift": round(float(out[2].item()), 6),
             "what": "bc_probe_drift over layer 0 (newest vs previous node)"}
+
+
+def time_sampling_loop(stream):
+    """Row f1: a whole 28-step flow sampler on the MMDiT workload (57 block outputs + the
+    velocity), equal-spaced schedule with N = 3 and K = 3.  Full steps: a stand-in model
+    (the seeded generator) writes every layer's new feature straight into the next cache slot,
+    the slot is committed, and the Euler step uses the written velocity; skipped steps: one
+    fused forecast + Euler launch over every layer.  Reports the device time of both kinds of
+    step; the stand-in's time says nothing about a real DiT."""
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    from paper_2608_28670_gb300 import synth
+    from paper_2608_28670_gb300.configs import WORKLOADS
+    from paper_2608_28670_gb300.runner import device_view
+    w = WORKLOADS["mmdit-t2i"]
+    K = w.K
+    ts = w.times() + [0.0]
+    sched = bc.bc_schedule_equal(w.steps, w.interval, K)
+    numels = w.numels
+    L = len(numels)
+    h = bc.bc_cache_create(numels, K, w.dtype)
+    try:
+        tdt = torch.bfloat16
+        outs = [torch.empty(w.layer_numel, dtype=tdt, device="cuda") for _ in range(w.n_layers)]
+        x = torch.zeros(numels[-1], dtype=torch.float32, device="cuda")
+        full_ms, skip_ms = [], []
+        for rep in range(2):                   # the first pass warms up
+            bc.bc_cache_reset(h)
+            full_ms, skip_ms = [], []
+            for i in range(w.steps):
+                t, dt = ts[i], ts[i + 1] - ts[i]
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                if sched[i]:
+                    slots = bc.bc_cache_next_slot_ptrs(h, L)
+                    for l, n in enumerate(numels):
+                        synth.fill_device(slots[l], w.dtype, n, seed=2026, tensor_id=l,
+                                          step_id=i, tau=t, degree=w.degree,
+                                          noise_std=w.noise_std, stream=stream)
+                    bc.bc_cache_commit(h, t)
+                    v = device_view(slots[-1], numels[-1], w.dtype).view(tdt)
+                    x.add_(v.float(), alpha=dt)
+                else:
+                    bc.bc_forecast_step(h, t, dt, [o.data_ptr() for o in outs] + [None],
+                                        w.dtype, L - 1, x.data_ptr(), bc.DTYPE_F32, stream)
+                b.record()
+                (full_ms if sched[i] else skip_ms).append((a, b))
+            torch.cuda.synchronize()
+        f = [a.elapsed_time(b) for a, b in full_ms]
+        sk = [a.elapsed_time(b) for a, b in skip_ms]
+        st = bc.bc_cache_stats(h)
+        return {"workload": "mmdit-t2i", "steps": w.steps, "full_steps": len(f),
+                "skipped_steps": len(sk), "skipped_step_ms": round(statistics.mean(sk), 4),
+                "skipped_total_ms": round(sum(sk), 3),
+                "standin_full_step_ms": round(statistics.mean(f), 4),
+                "forecast_GB/s": round(w.forecast_bytes(K, x_elem_bytes=4) /
+                                       (statistics.mean(sk) * 1e-3) / 1e9, 1),
+                "memo_hits": st["memo_hits"], "memo_misses": st["memo_misses"],
+                "what": "28-step flow sampler, equal-spaced N=3, K=3; full steps = seeded "
+                        "stand-in writing the next slot in place"}
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def time_blockwise(stream, steps):
+    """Row f2: a many-tensor (blockwise) cache -- 4096 tensors of 65,536 bf16 elements, K = 3
+    (1.6 GB of cache) -- forecast through per-layer output pointers (240 layers per launch)
+    and through one flat slot-shaped output (one launch)."""
+    import torch
+    from paper_2608_28670_gb300 import barycache as bc
+    from paper_2608_28670_gb300 import synth
+    n_t, n = 4096, 65536
+    numels = [n] * n_t
+    h = bc.bc_cache_create(numels, 3, bc.DTYPE_BF16)
+    try:
+        for j, t in enumerate((0.9, 0.85, 0.8)):
+            slots = bc.bc_cache_next_slot_ptrs(h, n_t)
+            offs = bc.bc_cache_layout(h, n_t)
+            synth.fill_device(slots[0], bc.DTYPE_BF16, offs[-1] // 2, seed=7, tensor_id=0,
+                              step_id=j, tau=t, degree=2, noise_std=1e-2, stream=stream)
+            bc.bc_cache_commit(h, t)
+        offs = bc.bc_cache_layout(h, n_t)
+        flat = torch.empty(offs[-1] // 2, dtype=torch.bfloat16, device="cuda")
+        per = [flat.data_ptr() + offs[l] for l in range(n_t)]
+        alg = (3 * 2 + 2) * n * n_t
+
+        def timed(fn):
+            for _ in range(3):
+                fn()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            a.record()
+            for _ in range(steps):
+                fn()
+            b.record()
+            torch.cuda.synchronize()
+            return a.elapsed_time(b) / steps
+        l0 = bc.bc_cache_stats(h)["kernel_launches"]
+        ms_layers = timed(lambda: bc.bc_forecast(h, 0.75, per, bc.DTYPE_BF16, stream))
+        l1 = bc.bc_cache_stats(h)["kernel_launches"]
+        ms_flat = timed(lambda: bc.bc_forecast_flat(h, 0.75, flat.data_ptr(), stream))
+        l2 = bc.bc_cache_stats(h)["kernel_launches"]
+        return {"tensors": n_t, "elements_per_tensor": n,
+                "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
+                              "ms": round(ms_layers, 4),
+                              "launches_per_call": (l1 - l0) // (steps + 3)},
+                "flat": {"GB/s": round(alg / (ms_flat * 1e-3) / 1e9, 1), "ms": round(ms_flat, 4),
+                         "launches_per_call": (l2 - l1) // (steps + 3)}}
+    finally:
+        bc.bc_cache_destroy(h)
 
 
 def time_fused(args, stream, dist):
