@@ -57,8 +57,10 @@ def _load():
     global _lib
     with _lock:
         if _lib is None:
-            build()
-            lib = ctypes.CDLL(_LIB)
+            # ORACLE_LIB points the pins at a deliberately broken build of oracle.c (the
+            # mutation test); normally the oracle is built from its source here.
+            path = os.environ.get("ORACLE_LIB") or build()
+            lib = ctypes.CDLL(path)
             dp = ctypes.POINTER(ctypes.c_double)
             lib.oracle_lagrange.argtypes = [dp, ctypes.c_int, ctypes.c_double, dp]
             lib.oracle_lagrange.restype = ctypes.c_int
