@@ -176,7 +176,8 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     torch.cuda.synchronize()
     if dist is not None:
         dist.barrier()
-    launches0 = run.stats()["kernel_launches"]
+    st0 = run.stats()
+    launches0 = st0["kernel_launches"]
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     host_s = []
@@ -192,8 +193,10 @@ def time_forecast(run, steps, warmup, stream, dist=None):
         dist.barrier()
     total_ms = starts[0].elapsed_time(ends[-1])
     per_step = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    launches = run.stats()["kernel_launches"] - launches0
+    st1 = run.stats()
+    launches = st1["kernel_launches"] - launches0
     time_forecast.host_us = 1e6 * statistics.median(host_s)
+    time_forecast.pipeline = st1["pipeline_launches"] - st0["pipeline_launches"]
     return total_ms, per_step, launches
 
 
@@ -266,7 +269,9 @@ def run_ours(args):
                 "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
                 "traffic": (round(traffic_per_elem * per_launch_elems)
                             if traffic_per_elem else None),
-                "kernel": "bc::forecast_kernel", "avg_launch_ms": round(kernel_ms, 4),
+                "kernel": ("bc::forecast_tma_kernel (TMA pipeline)"
+                           if time_forecast.pipeline == launches else "bc::forecast_kernel"),
+                "avg_launch_ms": round(kernel_ms, 4),
                 "algorithmic_bytes_per_launch": per_launch_bytes,
             },
             "gpu_launches": launches,

@@ -28,7 +28,11 @@
  *  - Host-side cache state (ring head, node times) changes when the call is made, so
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
  *    stream (or with the caller's own synchronisation).
- *  - No exception crosses the ABI; device code never traps or waits.
+ *  - No exception crosses the ABI and device code never traps.  The forecast kernel for
+ *    H <= 3 waits on its own shared-memory pipeline (TMA bulk copies completing on
+ *    mbarriers); every such wait gives up after about one second, records the failure in the
+ *    handle's device status word and returns, so the device never hangs: bc_cache_check
+ *    reports it.
  */
 #ifndef BARYCACHE_H
 #define BARYCACHE_H
@@ -51,7 +55,8 @@ typedef enum {
     BC_ERR_NOT_READY = 5,          /* forecast before any feature was pushed */
     BC_ERR_DUPLICATE_NODE = 6,     /* pushed t equals a timestep already in the window */
     BC_ERR_DEGENERATE_WEIGHTS = 7, /* Eq. 11 normaliser vanishes; run a full step instead */
-    BC_ERR_BAD_HANDLE = 8          /* null, destroyed or foreign handle */
+    BC_ERR_BAD_HANDLE = 8,         /* null, destroyed or foreign handle */
+    BC_ERR_DEVICE_TIMEOUT = 9      /* a forecast's pipeline wait ran out (bc_cache_check) */
 } bc_status;
 
 typedef enum { BC_DTYPE_F32 = 0, BC_DTYPE_BF16 = 1 } bc_dtype;
@@ -77,12 +82,20 @@ typedef struct {
 
 typedef struct bc_cache *bc_handle;
 
+/* Forecast kernel selection (bc_cache_set_kernel).  AUTO: the shared-memory pipeline (TMA
+ * bulk copies into a three-stage ring, one CTA per SM) for H <= 3 when the launch has at
+ * least 16 tiles of 8 Ki bf16 / 4 Ki fp32 elements per SM, else the register kernel (each
+ * thread holds its history loads in registers, two CTAs per SM).  REGISTER / PIPELINE pin
+ * one; H = 4 launches always use the register kernel.  Both compute the same bits. */
+typedef enum { BC_KERNEL_AUTO = 0, BC_KERNEL_REGISTER = 1, BC_KERNEL_PIPELINE = 2 } bc_kernel;
+
 typedef struct {
     int64_t forecasts;       /* successful forecast calls (every bc_forecast* variant) */
     int64_t pushes;          /* successful bc_cache_push / bc_cache_commit calls */
     int64_t kernel_launches; /* CUDA kernels this handle has launched */
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
+    int64_t pipeline_launches; /* of kernel_launches: forecasts run by the TMA pipeline kernel */
 } bc_stats;
 
 /* ---------------------------------------------------------------- host-only calls */
@@ -119,8 +132,8 @@ bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtyp
 /* Create the cache context H_t of Eq. 6 for `n_layers` tensors of numels[l] elements of
  * `dtype`, with history length K (1..BC_MAX_K).  Allocates, on the current device, one
  * arena of bc_cache_bytes_for(...) bytes and 16 KiB of reduction scratch for
- * bc_probe_drift (the only device allocations the library makes; freed by
- * bc_cache_destroy).  p == NULL uses the paper's defaults.  Blocks until the allocation is
+ * bc_probe_drift plus a status word (the only device allocations the library makes; freed
+ * by bc_cache_destroy).  p == NULL uses the paper's defaults.  Blocks until the allocation is
  * done.  Errors: INVALID_ARG, OOM, CUDA. */
 bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
                           const bc_params *p, bc_handle *out);
@@ -134,6 +147,9 @@ bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
 
 /* Replace the weight parameters (clears the weight memo). */
 bc_status bc_cache_set_params(bc_handle h, const bc_params *p);
+
+/* Pin the forecast kernel of this handle (bc_kernel; default AUTO). */
+bc_status bc_cache_set_kernel(bc_handle h, int kernel);
 
 /* Forget every pushed node (the arena keeps its bytes; nothing is enqueued). */
 bc_status bc_cache_reset(bc_handle h);
@@ -289,6 +305,20 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
  * different threads) race.  Errors: INVALID_ARG, ALIGNMENT, CUDA. */
 bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
                                  double *out, void *stream);
+
+/* Report device-side failures of this handle's forecast launches since the last check:
+ * BC_ERR_DEVICE_TIMEOUT if any launch gave up waiting for its shared-memory pipeline (its
+ * outputs may then be incomplete), else BC_OK.  Waits for all work on the device, reads and
+ * clears the handle's device status word.  Errors: BAD_HANDLE, CUDA, DEVICE_TIMEOUT. */
+bc_status bc_cache_check(bc_handle h);
+
+/* Test hook for failure detection (no production use): what = 1 makes the next forecast
+ * launch of this handle with H <= 3 run the pipeline kernel and leave the first stage of
+ * every CTA's pipeline unarmed,
+ * so that its bounded wait runs out (about one second) and the launch returns early with the
+ * status word set, which bc_cache_check then reports; what = 0 cancels a pending injection.
+ * Nothing is faulted: the copies that were issued complete and are drained. */
+bc_status bc_cache_inject_fault(bc_handle h, int what);
 
 /* Counters of this handle (see bc_stats). */
 bc_status bc_cache_stats(bc_handle h, bc_stats *out);

@@ -18,9 +18,10 @@ LIB_PATH = os.path.join(_PKG, "lib", "libbarycache.so")
 
 BC_MAX_K = 4
 OK, ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_OOM, ERR_CUDA, ERR_NOT_READY, \
-    ERR_DUPLICATE_NODE, ERR_DEGENERATE_WEIGHTS, ERR_BAD_HANDLE = range(9)
+    ERR_DUPLICATE_NODE, ERR_DEGENERATE_WEIGHTS, ERR_BAD_HANDLE, ERR_DEVICE_TIMEOUT = range(10)
 DTYPE_F32, DTYPE_BF16 = 0, 1
 MODE_EXACT, MODE_PAPER = 0, 1
+KERNEL_AUTO, KERNEL_REGISTER, KERNEL_PIPELINE = 0, 1, 2
 
 
 class BaryCacheError(RuntimeError):
@@ -43,7 +44,7 @@ class bc_adaptive(ctypes.Structure):
 class bc_stats(ctypes.Structure):
     _fields_ = [("forecasts", ctypes.c_int64), ("pushes", ctypes.c_int64),
                 ("kernel_launches", ctypes.c_int64), ("memo_hits", ctypes.c_int64),
-                ("memo_misses", ctypes.c_int64)]
+                ("memo_misses", ctypes.c_int64), ("pipeline_launches", ctypes.c_int64)]
 
 
 _lib = None
@@ -102,6 +103,9 @@ _SIGNATURES = {
                            ctypes.c_int),
     "bc_probe_drift": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                         ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p], ctypes.c_int),
+    "bc_cache_check": ([ctypes.c_void_p], ctypes.c_int),
+    "bc_cache_set_kernel": ([ctypes.c_void_p, ctypes.c_int], ctypes.c_int),
+    "bc_cache_inject_fault": ([ctypes.c_void_p, ctypes.c_int], ctypes.c_int),
     "bc_probe_drift_noalloc": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int,
                                 ctypes.c_void_p, ctypes.c_void_p], ctypes.c_int),
 }
@@ -328,3 +332,18 @@ def bc_probe_drift_noalloc(cur: int, prev: int, n: int, dtype: int, out: int,
     """bc_probe_drift without a handle or any device allocation (static library scratch)."""
     _check(lib().bc_probe_drift_noalloc(cur or None, prev or None, n, dtype, out or None,
                                         stream or None), "bc_probe_drift_noalloc")
+
+
+def bc_cache_check(h: int) -> None:
+    """Raise BaryCacheError(ERR_DEVICE_TIMEOUT) if a forecast launch gave up waiting."""
+    _check(lib().bc_cache_check(h), "bc_cache_check")
+
+
+def bc_cache_inject_fault(h: int, what: int = 1) -> None:
+    """Test hook: make the next forecast launch's pipeline wait run out (what = 1)."""
+    _check(lib().bc_cache_inject_fault(h, what), "bc_cache_inject_fault")
+
+
+def bc_cache_set_kernel(h: int, kernel: int) -> None:
+    """Pin the forecast kernel (KERNEL_AUTO, KERNEL_REGISTER or KERNEL_PIPELINE)."""
+    _check(lib().bc_cache_set_kernel(h, kernel), "bc_cache_set_kernel")

@@ -215,6 +215,9 @@ struct bc_cache {
     bc_stats stats{};
     std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
     double *probe_partials = nullptr;             // device scratch of bc_probe_drift
+    uint32_t *status = nullptr;                   // device status word of the forecast kernels
+    bool inject_next = false;                     // test hook (bc_cache_inject_fault)
+    int kernel = BC_KERNEL_AUTO;                  // bc_kernel
 
     char *slot_base(int slot) const { return arena + static_cast<uint64_t>(slot) * slot_bytes; }
     int slot_of_node(int j) const { return ((head - j) % K + K) % K; }  // j = 0 newest
@@ -353,13 +356,18 @@ bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dty
     plan.x_dtype = x_dtype;
     plan.x = x0;
     plan.z = up.z ? z0 : 0;
+    plan.status = h->status;
+    plan.inject = h->inject_next ? 1 : 0;
+    plan.kernel = h->kernel;
     plan.layers = entries.data();
     plan.n_layers = static_cast<int>(entries.size());
 
     if (plan.n_layers > 0) {
         DeviceGuard g(h->device);
         if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
-        const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches);
+        const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches,
+                                                &h->stats.pipeline_launches);
+        h->inject_next = false;
         if (err != cudaSuccess) return cuda_fail(err, "forecast launch");
     }
     ++h->stats.forecasts;
@@ -386,6 +394,7 @@ const char *bc_status_string(bc_status s) {
     case BC_ERR_DUPLICATE_NODE: return "timestep already in the cache window";
     case BC_ERR_DEGENERATE_WEIGHTS: return "weight normaliser vanishes";
     case BC_ERR_BAD_HANDLE: return "bad handle";
+    case BC_ERR_DEVICE_TIMEOUT: return "a device pipeline wait timed out";
     }
     return "unknown status";
 }
@@ -481,8 +490,12 @@ bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype d
         }
         {
             void *mem = nullptr;
-            cudaError_t e = cudaMalloc(&mem, sizeof(double) * 2 * bc::kProbeMaxCtas);
+            // reduction scratch followed by the 4-byte status word (padded to 256 bytes)
+            const size_t scratch = sizeof(double) * 2 * bc::kProbeMaxCtas;
+            cudaError_t e = cudaMalloc(&mem, scratch + 256);
+            if (e == cudaSuccess) e = cudaMemset(static_cast<char *>(mem) + scratch, 0, 256);
             if (e != cudaSuccess) {
+                if (mem) cudaFree(mem);
                 cudaGetLastError();
                 if (h->arena) cudaFree(h->arena);
                 delete h;
@@ -490,6 +503,7 @@ bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype d
                                                       : cuda_fail(e, "cudaMalloc");
             }
             h->probe_partials = static_cast<double *>(mem);
+            h->status = reinterpret_cast<uint32_t *>(static_cast<char *>(mem) + scratch);
         }
         {
             std::lock_guard<std::mutex> lk(g_registry_mu);
@@ -546,6 +560,16 @@ bc_status bc_cache_set_params(bc_handle h, const bc_params *p) {
     if (!params_valid(prm)) return fail(BC_ERR_INVALID_ARG, "invalid weight parameters");
     h->params = prm;
     h->memo.table.clear();
+    return BC_OK;
+}
+
+bc_status bc_cache_set_kernel(bc_handle h, int kernel) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (kernel != BC_KERNEL_AUTO && kernel != BC_KERNEL_REGISTER && kernel != BC_KERNEL_PIPELINE)
+        return fail(BC_ERR_INVALID_ARG, "unknown kernel choice %d", kernel);
+    h->kernel = kernel;
     return BC_OK;
 }
 
@@ -780,9 +804,14 @@ bc_status bc_forecast_flat(bc_handle h, double t_new, void *out, void *stream) {
             plan.euler_layer = -1;
             plan.layers = &e;
             plan.n_layers = 1;
+            plan.status = h->status;
+            plan.inject = h->inject_next ? 1 : 0;
+            plan.kernel = h->kernel;
             DeviceGuard g(h->device);
             if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
-            const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches);
+            const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches,
+                                                &h->stats.pipeline_launches);
+            h->inject_next = false;
             if (err != cudaSuccess) return cuda_fail(err, "forecast launch");
         }
         ++h->stats.forecasts;
@@ -870,6 +899,33 @@ bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, b
     int64_t launches = 0;
     const int err = bc::launch_drift_static(cur, prev, n, dtype, out, stream, &launches);
     if (err != cudaSuccess) return cuda_fail(err, "no-allocation drift");
+    return BC_OK;
+}
+
+bc_status bc_cache_check(bc_handle h) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    DeviceGuard g(h->device);
+    if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+    uint32_t word = 0;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpy(&word, h->status, sizeof word, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device status");
+    if (word == 0) return BC_OK;
+    e = cudaMemset(h->status, 0, sizeof word);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
+    return fail(BC_ERR_DEVICE_TIMEOUT,
+                "a forecast launch gave up waiting for its shared-memory pipeline (status 0x%x); "
+                "outputs of launches since the last check may be incomplete", word);
+}
+
+bc_status bc_cache_inject_fault(bc_handle h, int what) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (what != 0 && what != 1) return fail(BC_ERR_INVALID_ARG, "unknown fault %d", what);
+    h->inject_next = (what == 1);
     return BC_OK;
 }
 

@@ -65,6 +65,8 @@ struct ForecastArgs {
     int32_t x_bf16;           // sampler state dtype (and z's): 1 = bf16, 0 = f32
     uint64_t x;               // sampler state address
     uint64_t z;               // noise address (0: no noise term)
+    uint32_t *status;         // device status word: bit 0 = a pipeline wait timed out
+    int32_t inject;           // test hook: leave the first pipeline stage unarmed
     int64_t total_tiles;
     LayerEntry layer[CAP];
 };
@@ -81,6 +83,9 @@ struct LaunchPlan {
     bc_dtype x_dtype;
     uint64_t x;
     uint64_t z;
+    uint32_t *status;
+    int inject;
+    int kernel;               // bc_kernel choice: 0 auto, 1 register, 2 pipeline
     const LayerEntry *layers; // tile_end filled by the launcher
     int n_layers;
 };
@@ -94,8 +99,10 @@ inline int64_t tiles_for(int64_t numel, int elem_bytes, int vec_bytes, int tile_
 }
 
 // Enqueue the grouped forecast (one launch per CAP-sized group of layers).  Returns the
-// CUDA error of the last launch; *launches is incremented per launch.
-int launch_forecast(const LaunchPlan &plan, void *stream, int64_t *launches);
+// CUDA error of the last launch; *launches is incremented per launch, *pipeline_launches
+// per launch of the shared-memory pipeline kernel.
+int launch_forecast(const LaunchPlan &plan, void *stream, int64_t *launches,
+                    int64_t *pipeline_launches);
 
 // Probe drift reduction (bc_probe.cu): at most kProbeMaxCtas partial pairs of scratch.
 constexpr int kProbeMaxCtas = 1024;

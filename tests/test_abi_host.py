@@ -47,7 +47,7 @@ def test_version_and_status_strings():
     assert bc.bc_version() >= 10000
     L = bc.lib()
     seen = set()
-    for s in range(9):
+    for s in range(10):
         msg = L.bc_status_string(s).decode()
         assert msg and msg not in seen
         seen.add(msg)

@@ -115,3 +115,64 @@ def test_degenerate_weights_status():
             bc.ERR_DEGENERATE_WEIGHTS
     finally:
         bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("flat", [False, True])
+def test_pipeline_wait_timeout_is_reported_and_recovers(flat):
+    """Failure detection on the device: the test hook leaves each CTA's first pipeline stage
+    unarmed, so the forecast kernel's bounded wait runs out (about a second); the launch
+    returns, bc_cache_check reports BC_ERR_DEVICE_TIMEOUT once, and the next forecast on the
+    same handle and context is correct."""
+    import time
+    import numpy as np
+    import oracle
+    from paper_2608_28670_gb300 import synth
+    from tests.gpu_helpers import assert_close, to_device, to_host
+    numels = [100_000, 3 * 8192 + 5]
+    times = [0.9, 0.85, 0.8]
+    feats = synth.host_trajectories([(n,) for n in numels], times, dtype="bf16", seed=44)
+    h = bc.bc_cache_create(numels, 3, bc.DTYPE_BF16)
+    try:
+        for t, per in zip(times, feats):
+            dev = [to_device(f) for f in per]
+            bc.bc_cache_push(h, [d.data_ptr() for d in dev], t, s())
+            torch.cuda.synchronize()
+        bc.bc_cache_check(h)
+        offs = bc.bc_cache_layout(h, 2)
+        flat_out = torch.empty(offs[-1] // 2, dtype=torch.int16, device="cuda")
+        outs = [torch.empty(n, dtype=torch.int16, device="cuda") for n in numels]
+
+        def forecast():
+            if flat:
+                bc.bc_forecast_flat(h, 0.75, flat_out.data_ptr(), s())
+            else:
+                bc.bc_forecast(h, 0.75, [o.data_ptr() for o in outs], bc.DTYPE_BF16, s())
+
+        bc.bc_cache_inject_fault(h, 1)
+        t0 = time.perf_counter()
+        forecast()
+        assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
+        assert 0.5 < time.perf_counter() - t0 < 60.0
+        bc.bc_cache_check(h)                         # reported once, then clear
+        forecast()                                   # the handle and context still work
+        bc.bc_cache_check(h)
+        torch.cuda.synchronize()
+        W = oracle.paper_weights([0.8, 0.85, 0.9], 0.75)
+        nf = feats[::-1]
+        host_flat = to_host(flat_out, bc.DTYPE_BF16)
+        for l, n in enumerate(numels):
+            got = host_flat[offs[l] // 2: offs[l] // 2 + n] if flat else to_host(outs[l], bc.DTYPE_BF16)
+            ref, bound = oracle.combine([f[l] for f in nf], W)
+            assert_close(got, ref, bound, bc.DTYPE_BF16, f"after recovery, layer {l}")
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def test_check_is_clean_after_normal_launches_and_rejects_unknown_choices():
+    h = bc.bc_cache_create([4096], 2, bc.DTYPE_BF16)
+    try:
+        assert _status(bc.bc_cache_inject_fault, h, 7) == bc.ERR_INVALID_ARG
+        assert _status(bc.bc_cache_set_kernel, h, 3) == bc.ERR_INVALID_ARG
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)

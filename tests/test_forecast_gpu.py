@@ -32,13 +32,18 @@ def built():
     torch.cuda.set_device(0)
 
 
+KERNELS = [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE]
+KNAME = {bc.KERNEL_REGISTER: "register", bc.KERNEL_PIPELINE: "pipeline"}
+
+
 def run_case(numels, K, n_push, in_dt, out_dt, params, t_new, push_times, seed,
-             zero_copy=False, pad=64):
+             zero_copy=False, pad=64, kernel=bc.KERNEL_AUTO):
     shapes = [(n,) for n in numels]
     taus = list(push_times)
     feats = synth.host_trajectories(shapes, taus, dtype=DT_NAME[in_dt], degree=2,
                                     noise_std=1e-2, seed=seed)
     h = bc.bc_cache_create(numels, K, in_dt, params)
+    bc.bc_cache_set_kernel(h, kernel)
     try:
         for i in range(n_push):
             if zero_copy:
@@ -74,50 +79,90 @@ def run_case(numels, K, n_push, in_dt, out_dt, params, t_new, push_times, seed,
                 continue
             ref, bound = oracle.combine([f[l] for f in newest_first], W)
             assert_close(host[pad:pad + n], ref, bound, out_dt, f"layer {l} numel {n}")
+        bc.bc_cache_check(h)
         return h
     except Exception:
         bc.bc_cache_destroy(h)
         raise
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 @pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 @pytest.mark.parametrize("out_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 @pytest.mark.parametrize("K", [1, 2, 3, 4])
-def test_ragged_layers_all_dtypes(in_dt, out_dt, K):
+def test_ragged_layers_all_dtypes(in_dt, out_dt, K, kernel):
     times = [0.9 - 0.05 * i for i in range(K)]
     h = run_case(RAGGED, K, K, in_dt, out_dt, bc.make_params(), times[-1] - 0.05, times,
-                 seed=K * 10 + in_dt * 2 + out_dt)
+                 seed=K * 10 + in_dt * 2 + out_dt, kernel=kernel)
     bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 @pytest.mark.parametrize("K", [2, 3, 4])
 @pytest.mark.parametrize("mode", [bc.MODE_EXACT, bc.MODE_PAPER])
-def test_partial_and_rotating_window(K, mode):
+def test_partial_and_rotating_window(K, mode, kernel):
     # Fewer pushes than K (m < K), exactly K, and K + 3 (the ring has wrapped).
     for n_push in (1, K - 1, K, K + 3):
         if n_push < 1:
             continue
         times = [980.0 - 20.0 * i for i in range(n_push)]
         h = run_case([5000, 70_001], K, n_push, bc.DTYPE_BF16, bc.DTYPE_BF16,
-                     bc.make_params(mode=mode), times[-1] - 20.0, times, seed=n_push)
+                     bc.make_params(mode=mode), times[-1] - 20.0, times, seed=n_push,
+                     kernel=kernel)
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 @pytest.mark.parametrize("lam,delta,C", [(0.0, 0.0, 10.0), (0.5, 0.0, 10.0), (1.0, 0.0, 10.0),
                                          (0.0, 0.7, 2.0), (0.2, 1.0, 10.0)])
-def test_weight_parameters_flow_time(lam, delta, C):
+def test_weight_parameters_flow_time(lam, delta, C, kernel):
     # Flow-matching time in [0, 1]: the clip of Eq. 10 is active at this spacing.
     times = [1.0, 25 / 28, 22 / 28]
     h = run_case([33_333, 8192], 3, 3, bc.DTYPE_BF16, bc.DTYPE_F32,
-                 bc.make_params(lam=lam, delta=delta, clip_C=C), 21 / 28, times, seed=5)
+                 bc.make_params(lam=lam, delta=delta, clip_C=C), 21 / 28, times, seed=5,
+                 kernel=kernel)
     bc.bc_cache_destroy(h)
 
 
-def test_zero_copy_push():
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+def test_zero_copy_push(kernel):
     times = [0.8, 0.7, 0.6, 0.5, 0.4]
     h = run_case([12_345, 1, 65_536], 3, 5, bc.DTYPE_BF16, bc.DTYPE_BF16, bc.make_params(),
-                 0.35, times, seed=11, zero_copy=True)
+                 0.35, times, seed=11, zero_copy=True, kernel=kernel)
     bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("K", [1, 2, 3])
+@pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+@pytest.mark.parametrize("out_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+def test_register_and_pipeline_kernels_agree_bitwise(K, in_dt, out_dt):
+    # The two kernels apply the same fp32 FMA chain; only where the history bytes travel
+    # through differs, so every output and the updated latent must match bit for bit.
+    numels = RAGGED + [3 * 8192 * 8 + 17]
+    times = [0.9 - 0.05 * i for i in range(K)]
+    feats = synth.host_trajectories([(n,) for n in numels], times, dtype=DT_NAME[in_dt], seed=K)
+    h = bc.bc_cache_create(numels, K, in_dt)
+    try:
+        for t, per in zip(times, feats):
+            dev = [to_device(f) for f in per]
+            bc.bc_cache_push(h, [d.data_ptr() for d in dev], t, stream())
+            torch.cuda.synchronize()
+        x0 = torch.linspace(-3, 3, numels[-1], device="cuda")
+        results = []
+        for kern in KERNELS:
+            bc.bc_cache_set_kernel(h, kern)
+            outs = [empty_out(n, out_dt) for n in numels[:-1]]
+            x = x0.clone()
+            bc.bc_forecast_update(h, times[-1] - 0.05, 0.99, -0.05, 0.0,
+                                  [o.data_ptr() for o in outs] + [None], out_dt,
+                                  len(numels) - 1, x.data_ptr(), bc.DTYPE_F32, None, stream())
+            torch.cuda.synchronize()
+            results.append([o.cpu() for o in outs] + [x.cpu()])
+        bc.bc_cache_check(h)
+        for a, b in zip(*results):
+            assert torch.equal(a, b)
+    finally:
+        bc.bc_cache_destroy(h)
 
 
 def test_exact_mode_node_hit_returns_the_node():
@@ -189,10 +234,11 @@ def test_many_layers_use_several_launches():
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 @pytest.mark.parametrize("x_dt", [bc.DTYPE_F32, bc.DTYPE_BF16])
 @pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 @pytest.mark.parametrize("store_v", [False, True])
-def test_fused_euler_step(x_dt, in_dt, store_v):
+def test_fused_euler_step(x_dt, in_dt, store_v, kernel):
     numels = [8192 * 2 + 3, 262_144 + 5]   # a block output and a ragged "velocity"
     times = [1.0, 25 / 28, 22 / 28]
     t_new, dt = 21 / 28, -1 / 28
@@ -200,6 +246,7 @@ def test_fused_euler_step(x_dt, in_dt, store_v):
     x0 = synth.host_trajectories([(numels[1],)], [0.0], dtype=DT_NAME[x_dt], degree=0,
                                  noise_std=0.0, seed=22)[0][0]
     h = bc.bc_cache_create(numels, 3, in_dt)
+    bc.bc_cache_set_kernel(h, kernel)
     try:
         for t, per in zip(times, feats):
             dev = [to_device(f) for f in per]

@@ -25,9 +25,10 @@ def built():
     torch.cuda.set_device(0)
 
 
-def _cache_with(numels, times, in_dt, seed, K=3):
+def _cache_with(numels, times, in_dt, seed, K=3, kernel=bc.KERNEL_AUTO):
     feats = synth.host_trajectories([(n,) for n in numels], times, dtype=DT[in_dt], seed=seed)
     h = bc.bc_cache_create(numels, K, in_dt)
+    bc.bc_cache_set_kernel(h, kernel)
     for t, per in zip(times, feats):
         dev = [to_device(f) for f in per]
         bc.bc_cache_push(h, [d.data_ptr() for d in dev], t, stream())
@@ -35,15 +36,16 @@ def _cache_with(numels, times, in_dt, seed, K=3):
     return h, feats
 
 
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE])
 @pytest.mark.parametrize("kind", ["ddpm", "ddim0", "ddim1"])
 @pytest.mark.parametrize("x_dt", [bc.DTYPE_F32, bc.DTYPE_BF16])
 @pytest.mark.parametrize("with_z", [False, True])
-def test_update_matches_oracle(kind, x_dt, with_z):
+def test_update_matches_oracle(kind, x_dt, with_z, kernel):
     # DDIM-style integer timesteps; eps is the cached model output (layer 1).
     numels = [3 * 8192 + 11, 65_536 + 3]
     times = [980.0, 960.0, 940.0]
     t_new = 920.0
-    h, feats = _cache_with(numels, times, bc.DTYPE_BF16, seed=31)
+    h, feats = _cache_with(numels, times, bc.DTYPE_BF16, seed=31, kernel=kernel)
     try:
         betas = np.linspace(1e-4, 0.02, 1000)
         ab = np.cumprod(1 - betas)
@@ -92,12 +94,13 @@ def test_update_rejects_aliasing_and_bad_coefficients():
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE])
 @pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
-def test_flat_forecast_many_small_tensors(in_dt):
+def test_flat_forecast_many_small_tensors(in_dt, kernel):
     rng = np.random.default_rng(5)
     numels = [int(v) for v in rng.integers(1, 3000, 500)] + [0, 40_000]
     times = [0.9, 0.85, 0.8]
-    h, feats = _cache_with(numels, times, in_dt, seed=6)
+    h, feats = _cache_with(numels, times, in_dt, seed=6, kernel=kernel)
     try:
         offs = bc.bc_cache_layout(h, len(numels))
         assert offs[-1] * 3 == bc.bc_cache_bytes(h)
