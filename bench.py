@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip timing the workload's other history depths K")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-host-cap-gb", type=float, default=48.0,
+                    help="page-locked host memory for the e2e leg, shared by the node's ranks")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -303,7 +305,8 @@ def run_ours(args):
             result["sweep"] = sweep
             run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
         if not args.no_e2e:      # before the CPU leg, which loads the host memory system
-            result["e2e"] = e2e(run, args.e2e_steps, world, dist)
+            result["e2e"] = e2e(run, args.e2e_steps, world, dist,
+                                host_cap_bytes=args.e2e_host_cap_gb * 1e9)
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
             result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
         if not args.no_extra:
@@ -555,7 +558,7 @@ def pinned_host_buffer(nbytes):
     return arr, (lambda: cudart.cudaHostUnregister(arr.ctypes.data)), "cudaHostRegister"
 
 
-def e2e(run, steps, world, dist, chunk_layers=6):
+def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
     """Same metric through the public API with host buffers.  Per step: the new full-step
     features (one slot, every layer) are copied from pinned host memory into the next cache
     slot and committed (zero-copy push, Eq. 6), the following skipped step is forecast, and
@@ -579,15 +582,26 @@ def e2e(run, steps, world, dist, chunk_layers=6):
     if ob != eb:
         return {"unavailable": "e2e reuses the input buffer for the output: dtypes differ"}
     sizes = [n * eb for n in run.numels]
-    offs = np.cumsum([0] + sizes)
-    total = int(offs[-1])
-    host, release, kind = pinned_host_buffer(total)
+    total = int(sum(sizes))
+    # Page-locked host memory per rank is capped (48 GB shared by the ranks of one node):
+    # when a slot does not fit, layers cycle through a ring of host buffers, so every step
+    # still moves a whole slot each way over the host link.
+    cap = int(host_cap_bytes) // max(world, 1)
+    if total <= cap:
+        offs = np.cumsum([0] + sizes)
+        host_bytes = total
+    else:
+        per = max(sizes)
+        ring = max(1, cap // per)
+        offs = np.array([(l % ring) * per for l in range(len(sizes))] + [ring * per])
+        host_bytes = ring * per
+    host, release, kind = pinned_host_buffer(int(host_bytes))
     if host is None:
         return {"unavailable": kind}
     try:
         tdt = torch.bfloat16 if run.w.dtype == bc.DTYPE_BF16 else torch.float32
         L = len(run.numels)
-        hviews = [torch.from_numpy(host[offs[l]:offs[l + 1]]).view(tdt) for l in range(L)]
+        hviews = [torch.from_numpy(host[offs[l]:offs[l] + sizes[l]]).view(tdt) for l in range(L)]
         newest = bc.bc_cache_slot_ptrs(run.h, 0, L)
         for l, n in enumerate(run.numels):
             hviews[l].copy_(device_view(newest[l], n, run.w.dtype).view(tdt))
@@ -598,7 +612,33 @@ def e2e(run, steps, world, dist, chunk_layers=6):
         done_out = [None] * len(chunks)
         shared_outs = run.window < run.n_feat
 
+        ring_mode = host_bytes < total
+
+        def one_step_ring(i):
+            # Layers share host buffers: upload, forecast and read back one chunk at a time,
+            # in order on one stream, so no host buffer is read while it is being written.
+            t_full, t_target = _continuation(run, i)
+            slots = bc.bc_cache_next_slot_ptrs(run.h, L)
+            bc.bc_cache_commit(run.h, t_full)
+            with torch.cuda.stream(s_fc):
+                for c, ls in enumerate(chunks):
+                    for l in ls:
+                        device_view(slots[l], run.numels[l], run.w.dtype).view(tdt).copy_(
+                            hviews[l], non_blocking=True)
+                    ptrs = [None] * L
+                    for l in ls:
+                        ptrs[l] = run.outs[l - ls[0] if shared_outs else l].data_ptr()
+                    bc.bc_forecast(run.h, t_target, ptrs, run.out_dtype, s_fc.cuda_stream)
+                    for l in ls:
+                        hviews[l].copy_(run.outs[l - ls[0] if shared_outs else l],
+                                        non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(s_fc)
+                done_out[-1] = ev
+
         def one_step(i):
+            if ring_mode:
+                return one_step_ring(i)
             t_full, t_target = _continuation(run, i)
             slots = bc.bc_cache_next_slot_ptrs(run.h, L)
             landed = []
@@ -645,7 +685,8 @@ def e2e(run, steps, world, dist, chunk_layers=6):
         for i in range(steps):
             one_step(i + 1)
         for ev in done_out:
-            torch.cuda.current_stream().wait_event(ev)
+            if ev is not None:
+                torch.cuda.current_stream().wait_event(ev)
         b.record()
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
@@ -655,10 +696,12 @@ def e2e(run, steps, world, dist, chunk_layers=6):
                 "h2d_bytes_per_step": total,
                 "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
                 "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
-                "chunk_layers": cl, "host_memory": kind,
+                "chunk_layers": cl, "host_memory": kind, "host_buffer_bytes": int(host_bytes),
+                "overlapped": not ring_mode,
                 "path": "pinned host -> next cache slot (bc_cache_next_slot_ptrs + "
-                        "bc_cache_commit) -> bc_forecast per chunk -> pinned host, "
-                        "3 streams"}
+                        "bc_cache_commit) -> bc_forecast per chunk -> pinned host, " +
+                        ("pipelined over 3 streams" if not ring_mode else
+                         "one chunk at a time on one stream (host buffers shared by layers)")}
     finally:
         torch.cuda.synchronize()
         release()
