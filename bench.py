@@ -109,7 +109,10 @@ class ClockSampler:
              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
              "clocks_event_reasons.sw_power_cap")
         try:
-            idx = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[0] or "0"
+            vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+            local = int(os.environ.get("LOCAL_RANK", "0"))
+            ids = [v for v in vis.split(",") if v] if vis else []
+            idx = ids[local] if local < len(ids) else (ids[0] if ids else str(local))
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", idx, f"--query-gpu={q}", "--format=csv,noheader,nounits",

@@ -141,6 +141,11 @@ bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype d
 /* Free the arena (synchronises the device first so no enqueued work still reads it). */
 bc_status bc_cache_destroy(bc_handle h);
 
+/* Shape of this cache: number of layers, history length K and storage dtype (any of the
+ * output pointers may be NULL).  Every per-layer array a call takes or fills has exactly
+ * n_layers entries. */
+bc_status bc_cache_info(bc_handle h, int *n_layers, int *K, int *dtype);
+
 /* Device bytes held by this cache: the arena (the 16 KiB reduction scratch and host
  * bookkeeping are not counted). */
 bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);

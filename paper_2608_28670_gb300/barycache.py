@@ -64,6 +64,8 @@ _SIGNATURES = {
                          ctypes.POINTER(ctypes.c_void_p)], ctypes.c_int),
     "bc_cache_destroy": ([ctypes.c_void_p], ctypes.c_int),
     "bc_cache_bytes": ([ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)], ctypes.c_int),
+    "bc_cache_info": ([ctypes.c_void_p, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int),
+                       ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "bc_cache_set_params": ([ctypes.c_void_p, ctypes.POINTER(bc_params)], ctypes.c_int),
     "bc_cache_reset": ([ctypes.c_void_p], ctypes.c_int),
     "bc_cache_push": ([ctypes.c_void_p, ctypes.POINTER(ctypes.c_void_p), ctypes.c_double,
@@ -144,6 +146,22 @@ def _ptr_array(ptrs: Sequence[int | None]):
     return (ctypes.c_void_p * len(ptrs))(*[p if p else None for p in ptrs])
 
 
+def _layer_count(h: int) -> int:
+    n = ctypes.c_int()
+    _check(lib().bc_cache_info(h, ctypes.byref(n), None, None), "bc_cache_info")
+    return n.value
+
+
+def _layer_ptrs(h: int, ptrs: Sequence[int | None], where: str):
+    """Per-layer pointer array of exactly the cache's layer count (the C call reads that
+    many entries, so a shorter list must never reach it)."""
+    n = _layer_count(h)
+    if len(ptrs) != n:
+        raise BaryCacheError(ERR_INVALID_ARG, where,
+                             f"{len(ptrs)} pointers given for a cache of {n} layers")
+    return _ptr_array(ptrs)
+
+
 def _params(mode=MODE_PAPER, delta=0.0, lam=0.0, clip_C=10.0, eta=1e-12) -> bc_params:
     return bc_params(mode, delta, lam, clip_C, eta)
 
@@ -212,12 +230,21 @@ def bc_cache_reset(h: int) -> None:
     _check(lib().bc_cache_reset(h), "bc_cache_reset")
 
 
+def bc_cache_info(h: int) -> tuple[int, int, int]:
+    """(n_layers, K, dtype) of a cache."""
+    n, k, d = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(lib().bc_cache_info(h, ctypes.byref(n), ctypes.byref(k), ctypes.byref(d)),
+           "bc_cache_info")
+    return n.value, k.value, d.value
+
+
 def bc_cache_push(h: int, layer_ptrs: Sequence[int], t: float, stream: int = 0) -> None:
-    _check(lib().bc_cache_push(h, _ptr_array(layer_ptrs), float(t), stream or None),
-           "bc_cache_push")
+    _check(lib().bc_cache_push(h, _layer_ptrs(h, layer_ptrs, "bc_cache_push"), float(t),
+                               stream or None), "bc_cache_push")
 
 
-def bc_cache_next_slot_ptrs(h: int, n_layers: int) -> list[int]:
+def bc_cache_next_slot_ptrs(h: int, n_layers: int | None = None) -> list[int]:
+    n_layers = _layer_count(h)        # the array the C call fills has exactly this size
     out = (ctypes.c_void_p * n_layers)()
     _check(lib().bc_cache_next_slot_ptrs(h, out), "bc_cache_next_slot_ptrs")
     return [v or 0 for v in out]
@@ -234,7 +261,8 @@ def bc_cache_nodes(h: int) -> list[float]:
     return list(out[:m.value])
 
 
-def bc_cache_slot_ptrs(h: int, j: int, n_layers: int) -> list[int]:
+def bc_cache_slot_ptrs(h: int, j: int, n_layers: int | None = None) -> list[int]:
+    n_layers = _layer_count(h)
     out = (ctypes.c_void_p * n_layers)()
     _check(lib().bc_cache_slot_ptrs(h, j, out), "bc_cache_slot_ptrs")
     return [v or 0 for v in out]
@@ -249,14 +277,15 @@ def bc_coefficients(h: int, t_new: float) -> list[float]:
 
 def bc_forecast(h: int, t_new: float, out_ptrs: Sequence[int | None], out_dtype: int,
                 stream: int = 0) -> None:
-    _check(lib().bc_forecast(h, float(t_new), _ptr_array(out_ptrs), out_dtype,
+    _check(lib().bc_forecast(h, float(t_new), _layer_ptrs(h, out_ptrs, "bc_forecast"), out_dtype,
                              stream or None), "bc_forecast")
 
 
 def bc_forecast_step(h: int, t_new: float, dt: float, out_ptrs: Sequence[int | None],
                      out_dtype: int, v_layer: int, x: int, x_dtype: int,
                      stream: int = 0) -> None:
-    _check(lib().bc_forecast_step(h, float(t_new), float(dt), _ptr_array(out_ptrs), out_dtype,
+    _check(lib().bc_forecast_step(h, float(t_new), float(dt),
+                                  _layer_ptrs(h, out_ptrs, "bc_forecast_step"), out_dtype,
                                   v_layer, x or None, x_dtype, stream or None),
            "bc_forecast_step")
 
@@ -271,7 +300,8 @@ def bc_forecast_update(h: int, t_new: float, a: float, b: float, c: float,
                        out_ptrs: Sequence[int | None], out_dtype: int, v_layer: int, x: int,
                        x_dtype: int, z: int | None = None, stream: int = 0) -> None:
     _check(lib().bc_forecast_update(h, float(t_new), float(a), float(b), float(c),
-                                    _ptr_array(out_ptrs), out_dtype, v_layer, x or None,
+                                    _layer_ptrs(h, out_ptrs, "bc_forecast_update"), out_dtype,
+                                    v_layer, x or None,
                                     x_dtype, z or None, stream or None), "bc_forecast_update")
 
 
@@ -280,7 +310,8 @@ def bc_forecast_flat(h: int, t_new: float, out: int, stream: int = 0) -> None:
            "bc_forecast_flat")
 
 
-def bc_cache_layout(h: int, n_layers: int) -> list[int]:
+def bc_cache_layout(h: int, n_layers: int | None = None) -> list[int]:
+    n_layers = _layer_count(h)
     out = (ctypes.c_int64 * (n_layers + 1))()
     _check(lib().bc_cache_layout(h, out), "bc_cache_layout")
     return list(out)

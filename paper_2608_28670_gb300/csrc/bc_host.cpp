@@ -541,6 +541,16 @@ bc_status bc_cache_destroy(bc_handle h) {
     return rc;
 }
 
+bc_status bc_cache_info(bc_handle h, int *n_layers, int *K, int *dtype) {
+    t_last_error.clear();
+    bc_status s = check_handle(h);
+    if (s != BC_OK) return s;
+    if (n_layers) *n_layers = h->n_layers;
+    if (K) *K = h->K;
+    if (dtype) *dtype = static_cast<int>(h->dtype);
+    return BC_OK;
+}
+
 bc_status bc_cache_bytes(bc_handle h, int64_t *bytes) {
     t_last_error.clear();
     bc_status s = check_handle(h);

@@ -176,3 +176,26 @@ def test_check_is_clean_after_normal_launches_and_rejects_unknown_choices():
         bc.bc_cache_check(h)
     finally:
         bc.bc_cache_destroy(h)
+
+
+def test_binding_rejects_per_layer_lists_of_the_wrong_length():
+    # The C calls read exactly n_layers pointers; the binding must stop shorter lists.
+    h = bc.bc_cache_create([256, 512], 2, bc.DTYPE_F32)
+    try:
+        assert bc.bc_cache_info(h) == (2, 2, bc.DTYPE_F32)
+        x = torch.zeros(512, device="cuda")
+        assert _status_py(bc.bc_cache_push, h, [x.data_ptr()], 0.5, s()) == bc.ERR_INVALID_ARG
+        bc.bc_cache_push(h, [x.data_ptr(), x.data_ptr()], 0.5, s())
+        assert _status_py(bc.bc_forecast, h, 0.4, [x.data_ptr()], bc.DTYPE_F32, s()) == \
+            bc.ERR_INVALID_ARG
+        assert _status_py(bc.bc_forecast, h, 0.4, [None] * 3, bc.DTYPE_F32, s()) == \
+            bc.ERR_INVALID_ARG
+        assert len(bc.bc_cache_next_slot_ptrs(h)) == 2 and len(bc.bc_cache_layout(h)) == 3
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+def _status_py(fn, *args):
+    with pytest.raises(bc.BaryCacheError) as ei:
+        fn(*args)
+    return ei.value.status

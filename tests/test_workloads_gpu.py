@@ -73,6 +73,7 @@ def check_run(run: WorkloadRun, rng, calls=None):
             V = [gather(slot_ptrs[j][-1], nv, w.dtype, idx) for j in range(m)]
             x_ref, _, xb = oracle.euler(V, W, x_before.cpu().numpy(), p.dt)
             assert_close(run.x.cpu().numpy(), x_ref, xb, bc.DTYPE_F32, f"{w.name} Euler x")
+    bc.bc_cache_check(h)            # no forecast launch gave up waiting
 
 
 def test_c2i_256_every_element():
