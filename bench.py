@@ -326,6 +326,8 @@ def run_ours(args):
         result["sampling_loop"] = time_sampling_loop(stream)
         torch.cuda.empty_cache()
         result["blockwise"] = time_blockwise(stream, args.steps)
+        torch.cuda.empty_cache()
+        result["other_workloads"] = time_other_workloads(stream, args.steps)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -509,6 +511,44 @@ def time_blockwise(stream, steps):
                          "launches_per_call": (l2 - l1) // (steps + 3)}}
     finally:
         bc.bc_cache_destroy(h)
+
+
+def time_other_workloads(stream, steps):
+    """The remaining workloads: c2i-256 (9.4 MB per forecast, L2-resident, so L2 is flushed
+    by writing 512 MB before every timed launch, outside its event pair), c2i-512 (K = 4,
+    2.6 GB) and t2i-1024 (K = 3, 4.2 GB)."""
+    import torch
+    from paper_2608_28670_gb300.configs import WORKLOADS
+    from paper_2608_28670_gb300.runner import WorkloadRun
+    flush = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda")
+    out = {}
+    for name in ("c2i-256", "c2i-512", "t2i-1024"):
+        w = WORKLOADS[name]
+        r = WorkloadRun(w, stream=stream)
+        try:
+            for _ in range(3):
+                r.forecast()
+            ms = []
+            for i in range(steps):
+                if name == "c2i-256":
+                    flush.fill_(i & 0xFF)
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                r.forecast()
+                b.record()
+                torch.cuda.synchronize()
+                ms.append(a.elapsed_time(b))
+            m = statistics.median(ms)
+            st = r.stats()
+            out[name] = {"GB/s": round(r.algorithmic_bytes() / (m * 1e-3) / 1e9, 1),
+                         "us": round(1e3 * m, 1), "bytes": r.algorithmic_bytes(),
+                         "K": r.K, "pipeline_kernel": st["pipeline_launches"] > 0,
+                         "l2": "flushed before each launch" if name == "c2i-256"
+                               else "inputs larger than L2"}
+        finally:
+            r.close()
+    return out
 
 
 def time_fused(args, stream, dist):

@@ -1,0 +1,158 @@
+/*
+ * abi_client.c -- a plain C client of libbarycache.so, with no Python in between.
+ *
+ *   abi_client host     host-only calls (weights, footprints, schedules, errors): no GPU
+ *   abi_client device   one cache on the current GPU: allocate with cudaMalloc, push three
+ *                       full-step features, forecast, read back, and compare every element
+ *                       with the fp64 oracle (liboracle, linked for the check only)
+ *
+ * Exit status 0 on success; a failing check prints what failed and exits 1.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "barycache.h"
+
+/* The oracle's C entry points (test infrastructure). */
+int oracle_paper_weights(const double *s, int m, double t, double delta, double lambda, double C,
+                         double eta, double *W);
+void oracle_combine(int dtype, const void *const *F, int m, const double *W, int64_t n,
+                    double *out, double *bound);
+
+/* The few CUDA runtime calls the device check needs, declared here so that the client
+ * compiles with a plain C compiler against libcudart. */
+typedef int cudaError_t;
+extern cudaError_t cudaMalloc(void **p, size_t n);
+extern cudaError_t cudaFree(void *p);
+extern cudaError_t cudaMemcpy(void *dst, const void *src, size_t n, int kind);
+extern cudaError_t cudaDeviceSynchronize(void);
+#define H2D 1
+#define D2H 2
+
+static int failures = 0;
+#define CHECK(cond, ...)                                                     \
+    do {                                                                     \
+        if (!(cond)) {                                                       \
+            fprintf(stderr, "FAILED %s:%d: ", __FILE__, __LINE__);          \
+            fprintf(stderr, __VA_ARGS__);                                    \
+            fprintf(stderr, "\n");                                           \
+            ++failures;                                                      \
+        }                                                                    \
+    } while (0)
+
+static int host_checks(void) {
+    bc_params p;
+    bc_params_default(&p);
+    CHECK(p.mode == BC_MODE_PAPER && p.clip_C == 10.0, "defaults");
+
+    /* Exact mode: one step past three equispaced nodes is (3, -3, 1). */
+    double nodes[3] = {940.0, 960.0, 980.0}, c[3];
+    p.mode = BC_MODE_EXACT;
+    CHECK(bc_solve(nodes, 3, 920.0, &p, c) == BC_OK, "bc_solve exact");
+    CHECK(fabs(c[0] - 3) < 1e-12 && fabs(c[1] + 3) < 1e-12 && fabs(c[2] - 1) < 1e-12,
+          "exact weights %g %g %g", c[0], c[1], c[2]);
+
+    /* Paper mode against the oracle's independent implementation. */
+    bc_params_default(&p);
+    double w_ref[3];
+    CHECK(bc_solve(nodes, 3, 920.0, &p, c) == BC_OK, "bc_solve paper");
+    oracle_paper_weights(nodes, 3, 920.0, 0.95, 0.0, 10.0, 1e-12, w_ref);
+    for (int j = 0; j < 3; ++j) CHECK(fabs(c[j] - w_ref[j]) < 1e-12, "paper weight %d", j);
+
+    /* Footprint of the 60-layer video cache at K = 3 and the equal-spaced schedule. */
+    int64_t numels[60], bytes = 0;
+    for (int l = 0; l < 60; ++l) numels[l] = (int64_t)118800 * 3072;
+    CHECK(bc_cache_bytes_for(numels, 60, 3, BC_DTYPE_BF16, &bytes) == BC_OK &&
+              bytes == 131383296000LL, "footprint %lld", (long long)bytes);
+    uint8_t full[50];
+    int n_full = 0;
+    CHECK(bc_schedule_equal(50, 4, 2, full) == BC_OK, "schedule");
+    for (int i = 0; i < 50; ++i) n_full += full[i];
+    CHECK(n_full == 14, "full steps %d", n_full);
+
+    /* Errors come back as codes with a message. */
+    double dup[2] = {0.5, 0.5};
+    p.mode = BC_MODE_EXACT;
+    CHECK(bc_solve(dup, 2, 0.4, &p, c) == BC_ERR_DUPLICATE_NODE && bc_last_error()[0] != 0,
+          "duplicate nodes");
+    CHECK(bc_cache_bytes(NULL, &bytes) == BC_ERR_BAD_HANDLE, "null handle");
+    CHECK(strcmp(bc_status_string(BC_OK), "ok") == 0, "status string");
+    return failures;
+}
+
+/* bf16 bit pattern of a float (round to nearest even), for the test data. */
+static uint16_t to_bf16(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+static int device_checks(void) {
+    const int64_t n = 3 * 8192 * 16 + 77;   /* several tiles and a ragged tail */
+    const double times[3] = {0.9, 0.85, 0.8};
+    const double t_new = 0.75;
+    uint16_t *host[3];
+    void *dev_in = NULL, *dev_out = NULL;
+    bc_handle h = NULL;
+    for (int k = 0; k < 3; ++k) {
+        host[k] = (uint16_t *)malloc(n * sizeof(uint16_t));
+        for (int64_t e = 0; e < n; ++e) {
+            const double a = sin(0.001 * e), b = cos(0.0007 * e), q = 0.3 * sin(0.0003 * e);
+            host[k][e] = to_bf16((float)(a + b * times[k] + q * times[k] * times[k]));
+        }
+    }
+    CHECK(bc_cache_create(&n, 1, 3, BC_DTYPE_BF16, NULL, &h) == BC_OK, "create: %s",
+          bc_last_error());
+    CHECK(cudaMalloc(&dev_in, n * 2) == 0 && cudaMalloc(&dev_out, n * 2) == 0, "cudaMalloc");
+    for (int k = 0; k < 3 && !failures; ++k) {
+        CHECK(cudaMemcpy(dev_in, host[k], n * 2, H2D) == 0, "upload");
+        const void *ptrs[1] = {dev_in};
+        CHECK(bc_cache_push(h, ptrs, times[k], NULL) == BC_OK, "push: %s", bc_last_error());
+        cudaDeviceSynchronize();
+    }
+    void *outs[1] = {dev_out};
+    CHECK(bc_forecast(h, t_new, outs, BC_DTYPE_BF16, NULL) == BC_OK, "forecast: %s",
+          bc_last_error());
+    CHECK(bc_cache_check(h) == BC_OK, "device status");
+    uint16_t *got = (uint16_t *)malloc(n * 2);
+    CHECK(cudaMemcpy(got, dev_out, n * 2, D2H) == 0, "download");
+
+    double nodes[3] = {times[2], times[1], times[0]}, W[3];
+    oracle_paper_weights(nodes, 3, t_new, 0.95, 0.0, 10.0, 1e-12, W);
+    const void *F[3] = {host[2], host[1], host[0]};
+    double *ref = (double *)malloc(n * sizeof(double)), *bound = (double *)malloc(n * sizeof(double));
+    oracle_combine(1, F, 3, W, n, ref, bound);
+    int64_t bad = 0;
+    for (int64_t e = 0; e < n; ++e) {
+        uint32_t u = (uint32_t)got[e] << 16;
+        float g;
+        memcpy(&g, &u, sizeof g);
+        if (!(fabs((double)g - ref[e]) <= ldexp(1.0, -8) * bound[e])) ++bad;
+    }
+    CHECK(bad == 0, "%lld of %lld elements outside 2^-8 * sum |W||F|", (long long)bad,
+          (long long)n);
+    bc_stats st;
+    CHECK(bc_cache_stats(h, &st) == BC_OK && st.forecasts == 1 && st.pushes == 3, "stats");
+    bc_cache_destroy(h);
+    cudaFree(dev_in);
+    cudaFree(dev_out);
+    for (int k = 0; k < 3; ++k) free(host[k]);
+    free(got);
+    free(ref);
+    free(bound);
+    return failures;
+}
+
+int main(int argc, char **argv) {
+    if (argc < 2) return 2;
+    int rc = 0;
+    if (strcmp(argv[1], "host") == 0) rc = host_checks();
+    else if (strcmp(argv[1], "device") == 0) rc = device_checks();
+    else return 2;
+    printf("%s checks: %s\n", argv[1], rc ? "FAILED" : "ok");
+    return rc ? 1 : 0;
+}
