@@ -68,15 +68,26 @@ def measured_peak():
 KERNEL_CODE_END = "// ------------------------------------------------------------------ launch plumbing"
 
 
+def _code_only(src: bytes) -> bytes:
+    """Source text without comments or whitespace, so that editing a comment does not void
+    a stored measurement."""
+    import re
+    text = src.decode()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    return re.sub(r"\s+", "", text).encode()
+
+
 def kernel_source_hash() -> str:
-    """Hash of the forecast kernel's device code (bc_forecast.cu up to its host launch
-    plumbing) and of the shared layout header: a change there voids a stored ncu figure."""
+    """Hash of the forecast kernels' device code (bc_forecast.cu up to its host launch
+    plumbing) and of the shared layout header, comments and whitespace ignored: a change
+    there voids a stored ncu figure."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_28670_gb300", "csrc")
     with open(os.path.join(csrc, "bc_forecast.cu"), "rb") as fh:
-        h.update(fh.read().split(KERNEL_CODE_END.encode(), 1)[0])
+        h.update(_code_only(fh.read().split(KERNEL_CODE_END.encode(), 1)[0]))
     with open(os.path.join(csrc, "bc_internal.h"), "rb") as fh:
-        h.update(fh.read())
+        h.update(_code_only(fh.read()))
     return h.hexdigest()[:16]
 
 

@@ -3,27 +3,31 @@
 // Eq. 13 applies one weight vector W to the H cached features of every tensor:
 //     out[e] = sum_{j=1..H} W_j * F_j[e].
 // Per element that is H loads, H fused multiply-adds and one store: about 0.6-0.8 flop
-// per byte, far below any compute ridge, so the kernel is a pure HBM stream and tensor
+// per byte, far below any compute ridge, so the kernels are pure HBM streams and tensor
 // cores have no role.  The design goals are (1) every cache byte crosses HBM exactly once,
-// (2) enough independent 16-byte loads in flight per SM to cover HBM latency, and (3) one
-// launch for all cached tensors, so a 60-layer forecast costs one kernel, not sixty.
+// (2) enough bytes in flight per SM to cover HBM latency, and (3) one launch for all cached
+// tensors, so a 60-layer forecast costs one kernel, not sixty.
 //
 // Work decomposition: every layer is cut into tiles of kThreads x VPT history vectors of
 // 32 bytes; tiles are numbered across layers by a prefix sum carried in the launch's
 // parameter block; a persistent grid splits the tile space into one contiguous range per
-// CTA, so every CTA streams sequential addresses.  For H <= 3 the history tiles are staged
-// through a three-stage shared-memory ring by TMA bulk copies (one CTA per SM); at H = 4
-// each thread instead issues all 16 of its 256-bit loads before using any (two CTAs per
-// SM), which measured faster there.
+// CTA, so every CTA streams sequential addresses.  Two kernels share the arithmetic
+// (combine_vector / combine_tail, so they produce the same bits) and differ in how the
+// history reaches the SM:
+//   forecast_tma_kernel  H <= 3: TMA bulk copies into a three-stage shared-memory ring,
+//                        one CTA per SM (7.33 TB/s at H = 3 on the 60-layer video
+//                        workload);
+//   forecast_kernel      H = 4 and small launches: every thread issues all of its 256-bit
+//                        loads into registers before using any, two CTAs per SM (7.24 TB/s
+//                        at H = 3, 7.21 at H = 4).
+// The path from 6.96 TB/s (128-bit register loads, three CTAs per SM, grid stride) to
+// these numbers came from sweeps of vector width, vectors per thread, CTA size and count,
+// cache hints, tile order, ring depth and store path on that workload.
 //
-// History loads are 256-bit ld.global.nc with L1::no_allocate (each byte is touched
-// once; the slots are 256-byte aligned); outputs, the Euler state and push sources carry
-// only the ABI's 16-byte alignment and use 128-bit (or 64-bit) accesses; stores are
-// st.global.cs (streaming).  A sweep over vector width, vectors per thread, CTA size and
-// CTAs per SM on the 60-layer video workload picked these values (7.18 TB/s at H = 3,
-// against 6.96 TB/s for 128-bit loads at three CTAs per SM).  Nothing here waits on another CTA, nothing
-// allocates, and nothing traps: out-of-range work is never issued because every vector
-// index is checked against the layer's length.
+// Outputs, the sampler state and push sources carry only the ABI's 16-byte alignment and
+// use 128-bit (or 64-bit) accesses; stores are st.global.cs (streaming).  No CTA waits on
+// another, nothing allocates and nothing traps: every vector index is checked against its
+// layer's length, and the pipeline kernel's waits on its own mbarriers are bounded.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
