@@ -161,6 +161,28 @@ class ClockSampler:
                 "power_w_max": max(r[2] for r in rows)}
 
 
+class nvtx_range:
+    """NVTX range around a bench phase (shows up in Nsight timelines); no-op without CUDA."""
+
+    def __init__(self, name: str):
+        self.name = name
+
+    def __enter__(self):
+        try:
+            import torch
+            torch.cuda.nvtx.range_push(self.name)
+            self.on = True
+        except Exception:
+            self.on = False
+        return self
+
+    def __exit__(self, *exc):
+        if self.on:
+            import torch
+            torch.cuda.nvtx.range_pop()
+        return False
+
+
 # ----------------------------------------------------------------------------- ranks
 def max_over_ranks(value: float, dist=None, device="cuda") -> float:
     """The slowest rank's value (time-like): all_reduce MAX, or the value itself at N = 1."""
@@ -187,9 +209,10 @@ def window_targets(w, K):
 def time_forecast(run, steps, warmup, stream, dist=None):
     import torch
     ts = window_targets(run.w, run.K)
-    for i in range(warmup):
-        run.forecast(ts[i % len(ts)])
-    torch.cuda.synchronize()
+    with nvtx_range("warmup"):
+        for i in range(warmup):
+            run.forecast(ts[i % len(ts)])
+        torch.cuda.synchronize()
     if dist is not None:
         dist.barrier()
     st0 = run.stats()
@@ -198,13 +221,14 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     host_s = []
     torch.cuda.synchronize()
-    for i in range(steps):
-        starts[i].record()
-        h0 = time.perf_counter()
-        run.forecast(ts[i % len(ts)])
-        host_s.append(time.perf_counter() - h0)
-        ends[i].record()
-    torch.cuda.synchronize()
+    with nvtx_range(f"timed {steps} skipped steps"):
+        for i in range(steps):
+            starts[i].record()
+            h0 = time.perf_counter()
+            run.forecast(ts[i % len(ts)])
+            host_s.append(time.perf_counter() - h0)
+            ends[i].record()
+        torch.cuda.synchronize()
     if dist is not None:
         dist.barrier()
     total_ms = starts[0].elapsed_time(ends[-1])
@@ -319,26 +343,34 @@ def run_ours(args):
             result["sweep"] = sweep
             run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
         if not args.no_e2e:      # before the CPU leg, which loads the host memory system
-            result["e2e"] = e2e(run, args.e2e_steps, world, dist,
-                                host_cap_bytes=args.e2e_host_cap_gb * 1e9)
+            with nvtx_range("e2e"):
+                result["e2e"] = e2e(run, args.e2e_steps, world, dist,
+                                    host_cap_bytes=args.e2e_host_cap_gb * 1e9)
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
-            result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
+            with nvtx_range("cpu_baseline"):
+                result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
         if not args.no_extra:
-            result["probe_drift"] = time_probe(run, args.steps)
-            result["push"] = time_push(run, args.steps)
+            with nvtx_range("probe_drift"):
+                result["probe_drift"] = time_probe(run, args.steps)
+            with nvtx_range("push"):
+                result["push"] = time_push(run, args.steps)
     finally:
         if run is not None:
             run.close()
     if not args.no_extra and w.name != "mmdit-t2i":
         torch.cuda.empty_cache()
-        result["fused_step"] = time_fused(args, stream, dist)
+        with nvtx_range("fused_step"):
+            result["fused_step"] = time_fused(args, stream, dist)
     if not args.no_extra:
         torch.cuda.empty_cache()
-        result["sampling_loop"] = time_sampling_loop(stream)
+        with nvtx_range("sampling_loop"):
+            result["sampling_loop"] = time_sampling_loop(stream)
         torch.cuda.empty_cache()
-        result["blockwise"] = time_blockwise(stream, args.steps)
+        with nvtx_range("blockwise"):
+            result["blockwise"] = time_blockwise(stream, args.steps)
         torch.cuda.empty_cache()
-        result["other_workloads"] = time_other_workloads(stream, args.steps)
+        with nvtx_range("other_workloads"):
+            result["other_workloads"] = time_other_workloads(stream, args.steps)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
