@@ -613,8 +613,7 @@ def time_fused(args, stream, dist):
 
 def pinned_host_buffer(nbytes):
     """Page-locked host memory of exactly `nbytes`: cudaHostAlloc through the CUDA runtime
-    that torch loaded (concurrent H2D + D2H on GB300 need it; registered pageable memory
-    serialises them), else cudaHostRegister of a numpy buffer.  Returns (uint8 array,
+    that torch loaded, else cudaHostRegister of a numpy buffer.  Returns (uint8 array,
     release function, description)."""
     import ctypes
     import glob
