@@ -558,37 +558,62 @@ def time_blockwise(stream, steps):
 
 def time_other_workloads(stream, steps):
     """The remaining workloads: c2i-256 (9.4 MB per forecast, L2-resident, so L2 is flushed
-    by writing 512 MB before every timed launch, outside its event pair), c2i-512 (K = 4,
-    2.6 GB) and t2i-1024 (K = 3, 4.2 GB)."""
+    by writing 512 MB before every timed launch, outside its event pair; the flush keeps the
+    device busy while the host enqueues the forecast), c2i-512 (K = 4, 2.6 GB) and t2i-1024
+    (K = 3, 4.2 GB), whose inputs exceed L2: `steps` forecasts back to back between one event
+    pair, as in the headline measurement.  `idle_start_us` is one call on an idle device
+    (host call to completion: memo lookup, table build and launch latency included)."""
     import torch
     from paper_2608_28670_gb300.configs import WORKLOADS
     from paper_2608_28670_gb300.runner import WorkloadRun
     flush = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda")
     out = {}
+
+    def pair():
+        return torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
     for name in ("c2i-256", "c2i-512", "t2i-1024"):
         w = WORKLOADS[name]
         r = WorkloadRun(w, stream=stream)
         try:
             for _ in range(3):
                 r.forecast()
-            ms = []
-            for i in range(steps):
-                if name == "c2i-256":
+            torch.cuda.synchronize()
+            if name == "c2i-256":
+                ms = []
+                for i in range(steps):
                     flush.fill_(i & 0xFF)
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
+                    a, b = pair()
+                    a.record()
+                    r.forecast()
+                    b.record()
+                    torch.cuda.synchronize()
+                    ms.append(a.elapsed_time(b))
+                m = statistics.median(ms)
+            else:
+                a, b = pair()
+                a.record()
+                for _ in range(steps):
+                    r.forecast()
+                b.record()
+                torch.cuda.synchronize()
+                m = a.elapsed_time(b) / steps
+            idle = []
+            for _ in range(5):
+                torch.cuda.synchronize()
+                a, b = pair()
                 a.record()
                 r.forecast()
                 b.record()
                 torch.cuda.synchronize()
-                ms.append(a.elapsed_time(b))
-            m = statistics.median(ms)
+                idle.append(a.elapsed_time(b))
             st = r.stats()
             out[name] = {"GB/s": round(r.algorithmic_bytes() / (m * 1e-3) / 1e9, 1),
                          "us": round(1e3 * m, 1), "bytes": r.algorithmic_bytes(),
+                         "idle_start_us": round(1e3 * statistics.median(idle), 1),
                          "K": r.K, "pipeline_kernel": st["pipeline_launches"] > 0,
                          "l2": "flushed before each launch" if name == "c2i-256"
-                               else "inputs larger than L2"}
+                               else "inputs larger than L2, launches back to back"}
         finally:
             r.close()
     return out

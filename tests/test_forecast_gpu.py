@@ -21,7 +21,7 @@ from tests.gpu_helpers import (as_f64, assert_close, device_view, empty_out, ora
 pytestmark = pytest.mark.gpu
 
 DT_NAME = {bc.DTYPE_F32: "f32", bc.DTYPE_BF16: "bf16"}
-# kTileVecs = 1024 vectors of 16 B: 8192 bf16 / 4096 f32 elements per tile.
+# A tile holds 16 KiB of each history slot (32 KiB at K = 4): 8192 bf16 / 4096 f32 elements.
 RAGGED = [1, 7, 8, 9, 4095, 4096, 4097, 8191, 8192, 8193, 3 * 8192 + 5, 100_003]
 
 
