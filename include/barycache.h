@@ -24,7 +24,15 @@
  *    library cannot check sizes of foreign allocations).
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  All
  *    device work is enqueued on it asynchronously; errors are reported by return value
- *    only, and no call blocks on the device except bc_cache_create/destroy.
+ *    only, and no call blocks on the device except bc_cache_create/destroy and
+ *    bc_cache_check.
+ *  - CUDA graphs: pushes, commits, forecasts (all variants) and the probe drift enqueue
+ *    kernels only (no allocation, copy or synchronisation), so they may be called while
+ *    `stream` is being captured.  The graph holds the slot addresses, weights and update
+ *    coefficients chosen when each call was made; replaying it repeats that device work
+ *    and does not move the handle's host state (ring head, node times, statistics).  The
+ *    first forecast of each kind on a device also queries and sets per-device kernel
+ *    attributes; run the loop once uncaptured before capturing it.
  *  - Host-side cache state (ring head, node times) changes when the call is made, so
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
  *    stream (or with the caller's own synchronisation).

@@ -1,0 +1,108 @@
+"""A whole sampling loop captured into one CUDA graph and replayed.
+
+Pushes (zero-copy slots and commits), forecasts and the fused DDIM update enqueue only
+kernels on the caller's stream (no allocation, copy or synchronisation), so a loop of them
+can be captured.  The graph holds the slot addresses and weights that the calls chose while
+it was captured; replaying it repeats that device work (the handle's host state does not
+move).  The replay must reproduce the eager loop bit for bit, every time, and the eager
+loop must match the fp64 oracle replayed step by step.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_28670_gb300 import barycache as bc
+from paper_2608_28670_gb300 import synth
+from tests.gpu_helpers import device_view
+
+pytestmark = pytest.mark.gpu
+
+STEPS, INTERVAL, K = 20, 3, 3
+NUMELS = [2 * 256 * 1152, 2 * 4 * 32 * 32]      # a block output + the eps prediction
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build_libraries()
+    torch.cuda.set_device(0)
+
+
+def schedule():
+    ts = [980.0 - 20.0 * i for i in range(STEPS)]
+    betas = np.linspace(1e-4, 0.02, 1000)
+    ab = np.cumprod(1.0 - betas)
+    coef = []
+    for i in range(STEPS):
+        t, t_prev = int(ts[i]), int(ts[i]) - 20
+        coef.append(bc.bc_ddim_coefficients(ab[t], ab[t_prev] if t_prev >= 0 else 1.0, 0.0))
+    return ts, coef
+
+
+def run_loop(h, x, out, sched, ts, coef, s):
+    """One DDIM sampling run: full steps have the stand-in write both layers into the next
+    slot and take the DDIM step from the written eps; skipped steps forecast both layers and
+    take the fused DDIM step."""
+    for i in range(STEPS):
+        a, b, _ = coef[i]
+        if sched[i]:
+            slots = bc.bc_cache_next_slot_ptrs(h, 2)
+            for l, n in enumerate(NUMELS):
+                synth.fill_device(slots[l], bc.DTYPE_F32, n, seed=5, tensor_id=l, step_id=i,
+                                  tau=ts[i] / 1000.0, degree=2, noise_std=1e-3, stream=s)
+            bc.bc_cache_commit(h, ts[i])
+            x.mul_(a).add_(device_view(slots[1], NUMELS[1], bc.DTYPE_F32), alpha=b)
+        else:
+            bc.bc_forecast_update(h, ts[i], a, b, 0.0, [out.data_ptr(), None], bc.DTYPE_F32, 1,
+                                  x.data_ptr(), bc.DTYPE_F32, None, s)
+
+
+def test_graph_replay_equals_eager_loop_and_oracle():
+    ts, coef = schedule()
+    sched = bc.bc_schedule_equal(STEPS, INTERVAL, K)
+    x0 = torch.linspace(-1.0, 1.0, NUMELS[1], device="cuda")
+    h = bc.bc_cache_create(NUMELS, K, bc.DTYPE_F32)
+    try:
+        out = torch.empty(NUMELS[0], device="cuda")
+        x = x0.clone()
+        s = torch.cuda.current_stream().cuda_stream
+        run_loop(h, x, out, sched, ts, coef, s)                # eager (also warms up)
+        torch.cuda.synchronize()
+        x_eager, out_eager = x.clone(), out.clone()
+
+        # fp64 oracle replay of the same loop from the generator's stored values
+        slot_hist, x_ref = [], x0.double().cpu().numpy()
+        for i in range(STEPS):
+            a, b, _ = coef[i]
+            if sched[i]:
+                v = torch.empty(NUMELS[1], device="cuda")
+                synth.fill_device(v.data_ptr(), bc.DTYPE_F32, NUMELS[1], seed=5, tensor_id=1,
+                                  step_id=i, tau=ts[i] / 1000.0, degree=2, noise_std=1e-3,
+                                  stream=s)
+                torch.cuda.synchronize()
+                slot_hist.append((ts[i], v.cpu().numpy()))
+                x_ref = a * x_ref + b * slot_hist[-1][1].astype(np.float64)
+            else:
+                win = slot_hist[-K:][::-1]
+                W = oracle.paper_weights([w[0] for w in win], ts[i])
+                v_hat, _ = oracle.combine([w[1] for w in win], W)
+                x_ref = a * x_ref + b * v_hat
+        np.testing.assert_allclose(x_eager.cpu().numpy(), x_ref, rtol=1e-4, atol=1e-4)
+
+        bc.bc_cache_reset(h)
+        g = torch.cuda.CUDAGraph()
+        x.copy_(x0)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            run_loop(h, x, out, sched, ts, coef, torch.cuda.current_stream().cuda_stream)
+        for _ in range(2):
+            x.copy_(x0)
+            out.zero_()
+            g.replay()
+            torch.cuda.synchronize()
+            assert torch.equal(x, x_eager)
+            assert torch.equal(out, out_eager)
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)
