@@ -595,8 +595,9 @@ def time_graph_loop(stream):
 
 def time_blockwise(stream, steps):
     """Row f2: a many-tensor (blockwise) cache -- 4096 tensors of 65,536 bf16 elements, K = 3
-    (1.6 GB of cache) -- forecast through per-layer output pointers (240 layers per launch)
+    (1.6 GB of cache) -- forecast through per-layer output pointers (1016 layers per launch)
     and through one flat slot-shaped output (one launch)."""
+    import numpy as np
     import torch
     from paper_2608_28670_gb300 import barycache as bc
     from paper_2608_28670_gb300 import synth
@@ -612,7 +613,7 @@ def time_blockwise(stream, steps):
             bc.bc_cache_commit(h, t)
         offs = bc.bc_cache_layout(h, n_t)
         flat = torch.empty(offs[-1] // 2, dtype=torch.bfloat16, device="cuda")
-        per = [flat.data_ptr() + offs[l] for l in range(n_t)]
+        per = np.array([flat.data_ptr() + offs[l] for l in range(n_t)], dtype=np.uint64)
         alg = (3 * 2 + 2) * n * n_t
 
         def timed(fn):
@@ -627,6 +628,12 @@ def time_blockwise(stream, steps):
             b.record()
             torch.cuda.synchronize()
             return a.elapsed_time(b) / steps
+        by_kernel = {}
+        for name, kern in (("register", bc.KERNEL_REGISTER), ("pipeline", bc.KERNEL_PIPELINE),
+                           ("auto", bc.KERNEL_AUTO)):
+            bc.bc_cache_set_kernel(h, kern)
+            by_kernel[name] = round(alg / (timed(
+                lambda: bc.bc_forecast(h, 0.75, per, bc.DTYPE_BF16, stream)) * 1e-3) / 1e9, 1)
         l0 = bc.bc_cache_stats(h)["kernel_launches"]
         ms_layers = timed(lambda: bc.bc_forecast(h, 0.75, per, bc.DTYPE_BF16, stream))
         l1 = bc.bc_cache_stats(h)["kernel_launches"]
@@ -635,7 +642,8 @@ def time_blockwise(stream, steps):
         return {"tensors": n_t, "elements_per_tensor": n,
                 "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
                               "ms": round(ms_layers, 4),
-                              "launches_per_call": (l1 - l0) // (steps + 3)},
+                              "launches_per_call": (l1 - l0) // (steps + 3),
+                              "GB/s_by_kernel": by_kernel},
                 "flat": {"GB/s": round(alg / (ms_flat * 1e-3) / 1e9, 1), "ms": round(ms_flat, 4),
                          "launches_per_call": (l2 - l1) // (steps + 3)}}
     finally:

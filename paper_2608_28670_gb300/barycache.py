@@ -13,6 +13,8 @@ import os
 import threading
 from typing import Sequence
 
+import numpy as np
+
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "lib", "libbarycache.so")
 
@@ -142,7 +144,14 @@ def _check(status: int, where: str) -> None:
         raise BaryCacheError(status, where, detail)
 
 
-def _ptr_array(ptrs: Sequence[int | None]):
+def _ptr_array(ptrs):
+    """A C array of device addresses.  A 1-D numpy array of uint64 / int64 addresses (0 for
+    NULL) is passed without a copy: for caches of thousands of tensors, converting a Python
+    list element by element costs far more host time than the forecast itself."""
+    if isinstance(ptrs, np.ndarray):
+        if ptrs.ndim != 1 or ptrs.dtype not in (np.uint64, np.int64):
+            raise TypeError("pointer arrays must be 1-D uint64 or int64")
+        return np.ascontiguousarray(ptrs).ctypes.data_as(ctypes.POINTER(ctypes.c_void_p))
     return (ctypes.c_void_p * len(ptrs))(*[p if p else None for p in ptrs])
 
 

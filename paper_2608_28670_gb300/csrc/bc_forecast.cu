@@ -213,6 +213,24 @@ __device__ __forceinline__ void store_scalar(char *base, int64_t e, float v) {
     }
 }
 
+// Place a layer cursor on the layer holding `tile`: a binary search over the tiles' prefix
+// sums (about ten dependent parameter loads for a full table, where a scan from layer 0
+// would take up to one per layer); `first` is the layer's first tile.
+template <int CAP>
+__device__ __forceinline__ void find_layer(const ForecastArgs<CAP> &a, int64_t tile, int &l,
+                                           int64_t &first) {
+    int lo = 0, hi = a.n_layers - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (tile < a.layer[mid].tile_end)
+            hi = mid;
+        else
+            lo = mid + 1;
+    }
+    l = lo;
+    first = lo > 0 ? a.layer[lo - 1].tile_end : 0;
+}
+
 // Advance the CTA's layer cursor so that `tile` lies in layer `l`.  Tiles only grow, so
 // the cursor only moves forward; `first` is the layer's first tile.
 template <int CAP>
@@ -323,11 +341,13 @@ __global__ void __launch_bounds__(kThreads)
 
     // Each CTA streams one contiguous range of tiles (better DRAM page locality than a
     // grid stride: 7.24 vs 7.18 TB/s on the video workload at H = 3).
-    int l = 0;
-    int64_t first = 0;
     const int64_t per_cta = (a.total_tiles + gridDim.x - 1) / gridDim.x;
     const int64_t t_lo = static_cast<int64_t>(blockIdx.x) * per_cta;
     const int64_t t_hi = t_lo + per_cta < a.total_tiles ? t_lo + per_cta : a.total_tiles;
+    if (t_lo >= t_hi) return;
+    int l;
+    int64_t first;
+    find_layer(a, t_lo, l, first);
     for (int64_t tile = t_lo; tile < t_hi; ++tile) {
         seek_layer(a, tile, l, first);
         const LayerEntry &L = a.layer[l];
@@ -482,11 +502,14 @@ __global__ void __launch_bounds__(kThreads)
         }
         ++issued;
     };
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 0 && t_lo < t_hi) {
+        find_layer(a, t_lo, pl, pfirst);
         for (int i = 0; i < S && t_lo + i < t_hi; ++i) issue(t_lo + i, i);
+    }
 
     int l = 0;
     int64_t first = 0;
+    if (t_lo < t_hi) find_layer(a, t_lo, l, first);
     for (int64_t tile = t_lo; tile < t_hi; ++tile) {
         const int64_t i = tile - t_lo;
         const int stage = static_cast<int>(i % S);
@@ -536,6 +559,7 @@ __global__ void __launch_bounds__(kThreads) copy_kernel(const __grid_constant__ 
     constexpr int EV = 16 / T::kBytes;
     int l = 0;
     int64_t first = 0;
+    if (blockIdx.x < a.total_tiles) find_layer(a, blockIdx.x, l, first);
     for (int64_t tile = blockIdx.x; tile < a.total_tiles; tile += gridDim.x) {
         seek_layer(a, tile, l, first);
         const LayerEntry &L = a.layer[l];
@@ -681,6 +705,9 @@ int launch_all(const LaunchPlan &p, cudaStream_t s, int64_t *launches, int64_t *
         if (n <= kLayersSmall)
             err = launch_group<K, TIn, TOut, kLayersSmall>(p, p.layers + base, n, eul, s, launches,
                                                            pipe);
+        else if (n <= kLayersMedium)
+            err = launch_group<K, TIn, TOut, kLayersMedium>(p, p.layers + base, n, eul, s,
+                                                            launches, pipe);
         else
             err = launch_group<K, TIn, TOut, kLayersLarge>(p, p.layers + base, n, eul, s, launches,
                                                            pipe);
@@ -720,6 +747,8 @@ int copy_all(const LayerEntry *layers, int n_layers, cudaStream_t s, int64_t *la
         const int n = n_layers - base < kLayersLarge ? n_layers - base : kLayersLarge;
         if (n <= kLayersSmall)
             err = copy_group<T, kLayersSmall>(layers + base, n, s, launches);
+        else if (n <= kLayersMedium)
+            err = copy_group<T, kLayersMedium>(layers + base, n, s, launches);
         else
             err = copy_group<T, kLayersLarge>(layers + base, n, s, launches);
     }

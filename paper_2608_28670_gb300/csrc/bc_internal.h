@@ -43,9 +43,12 @@ constexpr int kCopyVecsPerThread = 4;
 
 // Layers per launch carried in the kernel's parameter block.  The whole table travels as
 // a __grid_constant__ parameter, so a forecast needs no device-side scratch and no
-// host-to-device copy of its own; caches with more layers issue one launch per group.
+// host-to-device copy of its own; three table sizes keep the block small for the usual
+// few-dozen-layer caches, and caches with more than kLayersLarge layers issue one launch
+// per group.
 constexpr int kLayersSmall = 8;
-constexpr int kLayersLarge = 240;
+constexpr int kLayersMedium = 64;
+constexpr int kLayersLarge = 1016;
 
 struct LayerEntry {        // 32 bytes
     uint64_t src;          // forecast: byte offset of the layer in every slot;
@@ -70,6 +73,9 @@ struct ForecastArgs {
     int64_t total_tiles;
     LayerEntry layer[CAP];
 };
+
+// Kernel parameter blocks may hold up to 32,764 bytes (CUDA 12.1 and later).
+static_assert(sizeof(ForecastArgs<kLayersLarge>) <= 32764, "layer table exceeds the parameter block");
 
 // Host-side view of one launch, independent of CAP.
 struct LaunchPlan {

@@ -9,6 +9,7 @@ over windows of layers (NULL outputs elsewhere), reusing one window of output bu
 """
 from __future__ import annotations
 
+import numpy as np
 import torch
 
 from . import barycache as bc
@@ -58,6 +59,9 @@ class WorkloadRun:
             tdt = torch.float32 if self.out_dtype == bc.DTYPE_F32 else torch.bfloat16
             self.outs = [torch.empty(w.layer_numel, dtype=tdt, device="cuda")
                          for _ in range(self.window)]
+            # per-call output tables, built once (the binding passes numpy tables as is)
+            self._call_ptrs = [np.array([q or 0 for q in self.out_ptrs(c)], dtype=np.uint64)
+                               for c in range(self.calls)]
             self.x = None
             if self.euler:
                 nx = self.numels[-1]
@@ -99,7 +103,7 @@ class WorkloadRun:
         """One C-ABI call: the forecast of one window of layers (plus, on the first
         window, the fused Euler step on the velocity layer)."""
         t = self.problem.t if t is None else t
-        ptrs = self.out_ptrs(call)
+        ptrs = self._call_ptrs[call]
         if self.euler and call == 0:
             bc.bc_forecast_step(self.h, t, self.problem.dt, ptrs, self.out_dtype,
                                 len(self.numels) - 1, self.x.data_ptr(), bc.DTYPE_F32,

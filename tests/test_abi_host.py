@@ -274,3 +274,20 @@ def test_adaptive_schedule_accumulates_and_resets():
         bc.bc_adaptive_decide(st, float("nan"))
     with pytest.raises(bc.BaryCacheError):
         bc.bc_adaptive_init(-1.0, 2)
+
+
+def test_pointer_tables_from_lists_and_numpy_arrays():
+    # Both forms reach C as the same array of addresses (None / 0 = NULL); numpy tables are
+    # passed without a per-element conversion.
+    addrs = [16, None, 2 ** 40 + 32, 0]
+    want = [16, None, 2 ** 40 + 32, None]
+    p = bc._ptr_array(addrs)
+    assert [p[i] for i in range(4)] == want
+    for dt in (np.uint64, np.int64):
+        a = np.array([q or 0 for q in addrs], dtype=dt)
+        p = bc._ptr_array(a)
+        assert [p[i] for i in range(4)] == want
+    with pytest.raises(TypeError):
+        bc._ptr_array(np.array([16, 32], dtype=np.uint32))
+    with pytest.raises(TypeError):
+        bc._ptr_array(np.zeros((2, 2), dtype=np.uint64))

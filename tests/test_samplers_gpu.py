@@ -111,7 +111,7 @@ def test_flat_forecast_many_small_tensors(in_dt, kernel):
         bc.bc_forecast_flat(h, 0.75, flat.data_ptr(), stream())
         torch.cuda.synchronize()
         assert bc.bc_cache_stats(h)["kernel_launches"] - s0 == 1
-        # the per-layer path (three launches of <= 240 layers) gives the same bits
+        # the per-layer path (one launch with a 502-entry layer table) gives the same bits
         outs = [empty_out(n, in_dt) for n in numels]
         bc.bc_forecast(h, 0.75, [o.data_ptr() if n else None for o, n in zip(outs, numels)],
                        in_dt, stream())
