@@ -292,5 +292,14 @@ void oracle_drift(int dtype, const void *cur, const void *prev, int64_t n, doubl
     }
     out[0] = num;
     out[1] = den;
-    out[2] = den > 0.0 ? num / den : (num > 0.0 ? INFINITY : 0.0);
+    /* Relative change; a probe with no magnitude has ratio 0 (no change) or +inf (any
+     * change); a NaN anywhere in either tensor makes the ratio NaN. */
+    if (den > 0.0)
+        out[2] = num / den;
+    else if (den == 0.0 && num == 0.0)
+        out[2] = 0.0;
+    else if (den == 0.0 && num > 0.0)
+        out[2] = INFINITY;
+    else
+        out[2] = NAN;
 }

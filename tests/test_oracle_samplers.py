@@ -102,6 +102,11 @@ def test_drift_closed_forms():
     np.testing.assert_allclose(oracle.drift(cur, prev), [2.5, 15.0, 2.5 / 15.0])
     assert oracle.drift(np.ones(3, np.float32), np.zeros(3, np.float32))[2] == math.inf
     assert list(oracle.drift(np.zeros(3, np.float32), np.zeros(3, np.float32))) == [0, 0, 0]
+    # a NaN in either tensor poisons the ratio instead of reading as "no change"
+    nan3 = np.array([0.0, np.nan, 0.0], np.float32)
+    assert math.isnan(oracle.drift(np.zeros(3, np.float32), nan3)[2])
+    assert math.isnan(oracle.drift(nan3, np.zeros(3, np.float32))[2])
+    assert math.isnan(oracle.drift(nan3, np.ones(3, np.float32))[2])
     # scale invariance: scaling both tensors leaves the ratio unchanged
     rng = np.random.default_rng(0)
     a = rng.standard_normal(999).astype(np.float32)
