@@ -80,14 +80,15 @@ def _code_only(src: bytes) -> bytes:
 
 def kernel_source_hash() -> str:
     """Hash of the forecast kernels' device code (bc_forecast.cu up to its host launch
-    plumbing) and of the shared layout header, comments and whitespace ignored: a change
-    there voids a stored ncu figure."""
+    plumbing) and of the headers it includes from the package (layout, pipeline primitives),
+    comments and whitespace ignored: a change there voids a stored ncu figure."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_28670_gb300", "csrc")
     with open(os.path.join(csrc, "bc_forecast.cu"), "rb") as fh:
         h.update(_code_only(fh.read().split(KERNEL_CODE_END.encode(), 1)[0]))
-    with open(os.path.join(csrc, "bc_internal.h"), "rb") as fh:
-        h.update(_code_only(fh.read()))
+    for name in ("bc_internal.h", "bc_tma.cuh"):
+        with open(os.path.join(csrc, name), "rb") as fh:
+            h.update(_code_only(fh.read()))
     return h.hexdigest()[:16]
 
 

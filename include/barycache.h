@@ -37,10 +37,10 @@
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
  *    stream (or with the caller's own synchronisation).
  *  - No exception crosses the ABI and device code never traps.  The forecast kernel for
- *    H <= 3 waits on its own shared-memory pipeline (TMA bulk copies completing on
- *    mbarriers); every such wait gives up after about one second, records the failure in the
- *    handle's device status word and returns, so the device never hangs: bc_cache_check
- *    reports it.
+ *    H <= 3 and the large-probe drift kernel wait on their own shared-memory pipelines (TMA
+ *    bulk copies completing on mbarriers); every such wait gives up after about one second,
+ *    records the failure in the handle's device status word and returns, so the device
+ *    never hangs: bc_cache_check reports it.
  */
 #ifndef BARYCACHE_H
 #define BARYCACHE_H
@@ -90,11 +90,15 @@ typedef struct {
 
 typedef struct bc_cache *bc_handle;
 
-/* Forecast kernel selection (bc_cache_set_kernel).  AUTO: the shared-memory pipeline (TMA
- * bulk copies into a three-stage ring, one CTA per SM) for H <= 3 when the launch has at
- * least 16 tiles of 8 Ki bf16 / 4 Ki fp32 elements per SM, else the register kernel (each
- * thread holds its history loads in registers, two CTAs per SM).  REGISTER / PIPELINE pin
- * one; H = 4 launches always use the register kernel.  Both compute the same bits. */
+/* Kernel selection (bc_cache_set_kernel), for forecasts and the probe drift.  Forecasts,
+ * AUTO: the shared-memory pipeline (TMA bulk copies into a three-stage ring, one CTA per SM)
+ * for H <= 3 when the launch has at least 16 tiles of 8 Ki bf16 / 4 Ki fp32 elements per SM,
+ * else the register kernel (each thread holds its history loads in registers, two CTAs per
+ * SM); H = 4 launches always use the register kernel; both compute the same bits.  Probe
+ * drift, AUTO: the pipeline form (a five-stage ring of 16 KiB tiles of both tensors, one
+ * CTA per SM) from 16 such tiles per SM on, else register loads; the two forms group the
+ * partial sums differently, so they agree within rounding, not bit for bit.  REGISTER /
+ * PIPELINE pin one. */
 typedef enum { BC_KERNEL_AUTO = 0, BC_KERNEL_REGISTER = 1, BC_KERNEL_PIPELINE = 2 } bc_kernel;
 
 typedef struct {
@@ -103,7 +107,7 @@ typedef struct {
     int64_t kernel_launches; /* CUDA kernels this handle has launched */
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
-    int64_t pipeline_launches; /* of kernel_launches: forecasts run by the TMA pipeline kernel */
+    int64_t pipeline_launches; /* of kernel_launches: TMA pipeline kernels (forecast or drift) */
 } bc_stats;
 
 /* ---------------------------------------------------------------- host-only calls */
@@ -161,7 +165,7 @@ bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
 /* Replace the weight parameters (clears the weight memo). */
 bc_status bc_cache_set_params(bc_handle h, const bc_params *p);
 
-/* Pin the forecast kernel of this handle (bc_kernel; default AUTO). */
+/* Pin the kernel of this handle's forecasts and probe drifts (bc_kernel; default AUTO). */
 bc_status bc_cache_set_kernel(bc_handle h, int kernel);
 
 /* Forget every pushed node (the arena keeps its bytes; nothing is enqueued). */
@@ -291,11 +295,13 @@ bc_status bc_adaptive_decide(bc_adaptive *s, double drift, int *run_full);
 
 /* The probe drift of the adaptive schedule, on the device:
  *     out[0] = sum_e |cur[e] - prev[e]|,  out[1] = sum_e |prev[e]|,  out[2] = out[0]/out[1]
- * (out[2] = 0 when both sums are 0, +inf when only out[1] is).  cur, prev: device, n
+ * (out[2] = 0 when both sums are 0, +inf when only out[1] is, NaN when either sum is NaN).  cur, prev: device, n
  * elements of dtype, 16-byte aligned; out: 3 device doubles.  Two launches on `stream` with
- * a fixed reduction order (bitwise reproducible on one device), using the handle's
- * reduction scratch, so calls on one handle must not overlap on the device.  The caller
- * reads out[2] back to drive bc_adaptive_decide.  Errors: INVALID_ARG, ALIGNMENT, CUDA. */
+ * a fixed reduction order (bitwise reproducible on one device for a given kernel choice),
+ * using the handle's reduction scratch, so calls on one handle must not overlap on the
+ * device.  If the pipeline form gives up waiting (see bc_cache_check), out[] reads NaN.  The
+ * caller reads out[2] back to drive bc_adaptive_decide.  Errors: INVALID_ARG, ALIGNMENT,
+ * CUDA. */
 bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
                          bc_dtype dtype, double *out, void *stream);
 
@@ -319,18 +325,19 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
 bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
                                  double *out, void *stream);
 
-/* Report device-side failures of this handle's forecast launches since the last check:
- * BC_ERR_DEVICE_TIMEOUT if any launch gave up waiting for its shared-memory pipeline (its
- * outputs may then be incomplete), else BC_OK.  Waits for all work on the device, reads and
+/* Report device-side failures of this handle's forecast and drift launches since the last
+ * check: BC_ERR_DEVICE_TIMEOUT if any launch gave up waiting for its shared-memory pipeline
+ * (its outputs may then be incomplete), else BC_OK.  Waits for all work on the device, reads and
  * clears the handle's device status word.  Errors: BAD_HANDLE, CUDA, DEVICE_TIMEOUT. */
 bc_status bc_cache_check(bc_handle h);
 
 /* Test hook for failure detection (no production use): what = 1 makes the next forecast
  * launch of this handle with H <= 3 run the pipeline kernel and leave the first stage of
- * every CTA's pipeline unarmed,
- * so that its bounded wait runs out (about one second) and the launch returns early with the
- * status word set, which bc_cache_check then reports; what = 0 cancels a pending injection.
- * Nothing is faulted: the copies that were issued complete and are drained. */
+ * every CTA's pipeline unarmed, so that its bounded wait runs out (about one second) and the
+ * launch returns early with the status word set, which bc_cache_check then reports;
+ * what = 2 does the same to the next probe drift of at least one 16 KiB tile (its out[]
+ * then reads NaN); what = 0 cancels a pending injection.  Nothing is faulted: the copies
+ * that were issued complete and are drained. */
 bc_status bc_cache_inject_fault(bc_handle h, int what);
 
 /* Counters of this handle (see bc_stats). */

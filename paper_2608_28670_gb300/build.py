@@ -32,7 +32,8 @@ LIBS = {
     "libbarycache.so": ["bc_host.cpp", "bc_forecast.cu", "bc_probe.cu"],
     "libbc_synth.so": ["bc_synth.cu"],
 }
-HEADERS = [os.path.join(INCLUDE, "barycache.h"), os.path.join(CSRC, "bc_internal.h")]
+HEADERS = [os.path.join(INCLUDE, "barycache.h"), os.path.join(CSRC, "bc_internal.h"),
+           os.path.join(CSRC, "bc_tma.cuh")]
 
 
 def _newer(target: str, deps: list[str]) -> bool:

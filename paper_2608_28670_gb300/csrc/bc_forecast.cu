@@ -36,6 +36,7 @@
 #include <type_traits>
 
 #include "bc_internal.h"
+#include "bc_tma.cuh"
 
 namespace bc {
 namespace {
@@ -393,58 +394,7 @@ __global__ void __launch_bounds__(kThreads)
 // and returns, so a lost completion can never hang the device; the host reads the word
 // with bc_cache_check.
 constexpr int kTmaStages = 3;
-constexpr uint64_t kTmaWaitNs = 1000000000ull;
 constexpr int kTmaMinTilesPerCta = 16;
-
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint64_t global_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
-                 : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-                 "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Wait for the given phase parity; false if the time limit (or, as a backstop, an
-// iteration count) passed first.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_ns();
-    for (uint32_t spins = 0; !mbar_try_wait(bar, parity); ++spins)
-        if (global_ns() - t0 > kTmaWaitNs || spins > (1u << 26)) return false;
-    return true;
-}
-
-__device__ __forceinline__ void bulk_copy_to_shared(void *dst, const void *src, uint32_t bytes,
-                                                    uint64_t *bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-        ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
-        : "memory");
-}
 
 // Bytes of one history tile, and of the whole ring (kTmaStages stages of K tiles).
 template <int K>
@@ -472,7 +422,7 @@ __global__ void __launch_bounds__(kThreads)
     const int64_t t_hi = t_lo + per_cta < a.total_tiles ? t_lo + per_cta : a.total_tiles;
     if (threadIdx.x == 0) {
         for (int i = 0; i < S; ++i) mbar_init(&full[i], 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_init_fence();
         abort_flag = 0;
     }
     __syncthreads();

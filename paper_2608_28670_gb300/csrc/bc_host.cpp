@@ -216,7 +216,8 @@ struct bc_cache {
     std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
     double *probe_partials = nullptr;             // device scratch of bc_probe_drift
     uint32_t *status = nullptr;                   // device status word of the forecast kernels
-    bool inject_next = false;                     // test hook (bc_cache_inject_fault)
+    bool inject_next = false;                     // test hooks (bc_cache_inject_fault):
+    bool inject_next_drift = false;               //   next forecast / next probe drift
     int kernel = BC_KERNEL_AUTO;                  // bc_kernel
 
     char *slot_base(int slot) const { return arena + static_cast<uint64_t>(slot) * slot_bytes; }
@@ -886,8 +887,11 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
         return fail(BC_ERR_ALIGNMENT, "probe tensors must be 16-byte aligned");
     DeviceGuard g(h->device);
     if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+    bc::DriftOptions opt{h->kernel, h->status, h->inject_next_drift ? 1 : 0};
     const int err = bc::launch_drift(cur, prev, n, dtype, h->probe_partials, bc::kProbeMaxCtas,
-                                     out, stream, &h->stats.kernel_launches);
+                                     out, opt, stream, &h->stats.kernel_launches,
+                                     &h->stats.pipeline_launches);
+    h->inject_next_drift = false;
     if (err != cudaSuccess) return cuda_fail(err, "drift launch");
     return BC_OK;
 }
@@ -926,7 +930,7 @@ bc_status bc_cache_check(bc_handle h) {
     e = cudaMemset(h->status, 0, sizeof word);
     if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
     return fail(BC_ERR_DEVICE_TIMEOUT,
-                "a forecast launch gave up waiting for its shared-memory pipeline (status 0x%x); "
+                "a launch gave up waiting for its shared-memory pipeline (status 0x%x); "
                 "outputs of launches since the last check may be incomplete", word);
 }
 
@@ -934,8 +938,9 @@ bc_status bc_cache_inject_fault(bc_handle h, int what) {
     t_last_error.clear();
     bc_status s = check_handle(h);
     if (s != BC_OK) return s;
-    if (what != 0 && what != 1) return fail(BC_ERR_INVALID_ARG, "unknown fault %d", what);
+    if (what < 0 || what > 2) return fail(BC_ERR_INVALID_ARG, "unknown fault %d", what);
     h->inject_next = (what == 1);
+    h->inject_next_drift = (what == 2);
     return BC_OK;
 }
 

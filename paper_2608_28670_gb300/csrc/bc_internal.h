@@ -113,10 +113,19 @@ int launch_forecast(const LaunchPlan &plan, void *stream, int64_t *launches,
 // Probe drift reduction (bc_probe.cu): at most kProbeMaxCtas partial pairs of scratch.
 constexpr int kProbeMaxCtas = 1024;
 int probe_ctas();
+// The handle's side of a drift launch: kernel choice (bc_kernel), device status word and
+// the test hook that leaves the pipeline's first stage unarmed.
+struct DriftOptions {
+    int kernel;
+    uint32_t *status;
+    int inject;
+};
 // Enqueue sum |cur - prev|, sum |prev| and their ratio into out[0..2] (device doubles),
-// using partials[0 .. 2 * max_parts) as scratch.  Two launches.
+// using partials[0 .. 2 * max_parts) as scratch.  Two launches; *pipeline_launches counts
+// the shared-memory pipeline variant of the first.
 int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, double *partials,
-                 int max_parts, double *out, void *stream, int64_t *launches);
+                 int max_parts, double *out, const DriftOptions &opt, void *stream,
+                 int64_t *launches, int64_t *pipeline_launches);
 
 // The no-allocation drift (bc_probe.cu): scratch is a file-scope device array of
 // kStaticDriftMaxTiles partial pairs (256 KiB), one pair per tile of

@@ -1,0 +1,76 @@
+// bc_tma.cuh -- the shared-memory pipeline primitives of the streaming kernels (sm_103a):
+// 1-D TMA bulk copies (cp.async.bulk, global -> shared) completing on mbarriers with a
+// transaction count, and mbarrier waits bounded in time.
+//
+// A stage's mbarrier is initialised with one arrival; the producer thread arms it with
+// mbarrier.arrive.expect_tx (the bytes the stage will receive) and issues the bulk copies,
+// whose completion decrements the transaction count; the phase flips when both are done.
+// Waiters spin on mbarrier.try_wait.parity with a limit of kTmaWaitNs by %globaltimer (and
+// an iteration backstop), so a completion that never comes ends in a reported failure,
+// never in a hung device.
+#pragma once
+
+#include <cstdint>
+
+namespace bc {
+
+constexpr uint64_t kTmaWaitNs = 1000000000ull;   // about one second
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+                 : "memory");
+}
+
+// Make the initialised barriers visible to the async proxy (the bulk copies).
+__device__ __forceinline__ void mbar_init_fence() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the given phase parity; false if the time limit (or, as a backstop, an
+// iteration count) passed first.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t spins = 0; !mbar_try_wait(bar, parity); ++spins)
+        if (global_ns() - t0 > kTmaWaitNs || spins > (1u << 26)) return false;
+    return true;
+}
+
+// Copy `bytes` (a multiple of 16; both addresses 16-byte aligned) from global to shared
+// memory, completing on `bar`.
+__device__ __forceinline__ void bulk_copy_to_shared(void *dst, const void *src, uint32_t bytes,
+                                                    uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+}  // namespace bc

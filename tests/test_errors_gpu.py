@@ -168,10 +168,43 @@ def test_pipeline_wait_timeout_is_reported_and_recovers(flat):
         bc.bc_cache_destroy(h)
 
 
+def test_drift_pipeline_wait_timeout_is_reported_and_recovers():
+    """The same failure detection for the probe drift's pipeline form: with its first stage
+    left unarmed every CTA gives up, out[] reads NaN, bc_cache_check reports the timeout once,
+    and the next drift on the handle is right."""
+    import time
+    import numpy as np
+    import oracle
+    from tests.gpu_helpers import to_device
+    n = 8192 * 300 + 5
+    rng = np.random.default_rng(3)
+    prev = rng.standard_normal(n).astype(np.float32)
+    cur = prev + 0.1 * rng.standard_normal(n).astype(np.float32)
+    c, p = to_device(cur), to_device(prev)
+    h = bc.bc_cache_create([16], 2, bc.DTYPE_F32)
+    bc.bc_cache_set_kernel(h, bc.KERNEL_PIPELINE)
+    try:
+        out = torch.zeros(3, dtype=torch.float64, device="cuda")
+        bc.bc_cache_inject_fault(h, 2)
+        t0 = time.perf_counter()
+        bc.bc_probe_drift(h, c.data_ptr(), p.data_ptr(), n, bc.DTYPE_F32, out.data_ptr(), s())
+        assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
+        assert 0.5 < time.perf_counter() - t0 < 60.0
+        assert np.isnan(out.cpu().numpy()).all()
+        bc.bc_cache_check(h)
+        bc.bc_probe_drift(h, c.data_ptr(), p.data_ptr(), n, bc.DTYPE_F32, out.data_ptr(), s())
+        bc.bc_cache_check(h)
+        np.testing.assert_allclose(out.cpu().numpy(), oracle.drift(cur, prev), rtol=2e-6)
+        assert bc.bc_cache_stats(h)["pipeline_launches"] == 2
+    finally:
+        bc.bc_cache_destroy(h)
+
+
 def test_check_is_clean_after_normal_launches_and_rejects_unknown_choices():
     h = bc.bc_cache_create([4096], 2, bc.DTYPE_BF16)
     try:
         assert _status(bc.bc_cache_inject_fault, h, 7) == bc.ERR_INVALID_ARG
+        assert _status(bc.bc_cache_inject_fault, h, -1) == bc.ERR_INVALID_ARG
         assert _status(bc.bc_cache_set_kernel, h, 3) == bc.ERR_INVALID_ARG
         bc.bc_cache_check(h)
     finally:

@@ -146,15 +146,22 @@ def test_flat_forecast_rejects_bad_output():
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE],
+                         ids=["register", "pipeline"])
 @pytest.mark.parametrize("dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
-@pytest.mark.parametrize("n", [0, 1, 7, 8, 9, 1000, 123_457, 4 * 1024 * 1024 + 3])
-def test_probe_drift_matches_oracle_and_is_deterministic(dt, n):
+@pytest.mark.parametrize("n", [0, 1, 7, 8, 9, 1000, 123_457, 8192 * 37 + 11,
+                               4 * 1024 * 1024 + 3])
+def test_probe_drift_matches_oracle_and_is_deterministic(dt, n, kernel):
+    # The pipeline form stages 16 KiB tiles of both tensors (8192 bf16 / 4096 fp32
+    # elements); these sizes give one partial tile, many tiles with a ragged last one, and
+    # an element tail shorter than one 16-byte group.
     rng = np.random.default_rng(n + dt)
     prev = rng.standard_normal(n).astype(np.float32)
     cur = prev + 0.05 * rng.standard_normal(n).astype(np.float32)
     if dt == bc.DTYPE_BF16:
         prev, cur = synth.f32_to_bf16_bits(prev), synth.f32_to_bf16_bits(cur)
     h = bc.bc_cache_create([16], 2, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
     try:
         c, p = to_device(cur), to_device(prev)
         out = torch.full((2, 3), -1.0, dtype=torch.float64, device="cuda")
@@ -168,12 +175,16 @@ def test_probe_drift_matches_oracle_and_is_deterministic(dt, n):
             assert list(got[0]) == [0.0, 0.0, 0.0]
         else:
             np.testing.assert_allclose(got[0], ref, rtol=2e-6)
+        bc.bc_cache_check(h)
     finally:
         bc.bc_cache_destroy(h)
 
 
-def test_probe_drift_special_values():
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE],
+                         ids=["register", "pipeline"])
+def test_probe_drift_special_values(kernel):
     h = bc.bc_cache_create([16], 2, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
     try:
         z = torch.zeros(1000, device="cuda")
         o = torch.ones(1000, device="cuda")
@@ -186,6 +197,12 @@ def test_probe_drift_special_values():
                           stream())
         torch.cuda.synchronize()
         assert out.cpu().tolist() == [0.0, 1000.0, 0.0]
+        zn = z.clone()
+        zn[500] = float("nan")
+        bc.bc_probe_drift(h, z.data_ptr(), zn.data_ptr(), 1000, bc.DTYPE_F32, out.data_ptr(),
+                          stream())
+        torch.cuda.synchronize()
+        assert np.isnan(out.cpu().numpy()).all()        # NaN, never "no change"
         with pytest.raises(bc.BaryCacheError) as ei:
             bc.bc_probe_drift(h, o.data_ptr() + 4, z.data_ptr(), 10, bc.DTYPE_F32,
                               out.data_ptr(), stream())
