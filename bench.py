@@ -402,19 +402,28 @@ def time_push(run, steps):
         return None
     ptrs = [o.data_ptr() for o in run.outs]
     slot = sum(n * run.w.elem_bytes for n in run.numels)
-    t = [_continuation(run, 100 + i)[0] for i in range(steps + 2)]
-    for i in range(2):
-        bc.bc_cache_push(run.h, ptrs, t[i], run.stream)
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    a.record()
-    for i in range(steps):
-        bc.bc_cache_push(run.h, ptrs, t[2 + i], run.stream)
-    b.record()
-    torch.cuda.synchronize()
-    ms = a.elapsed_time(b) / steps
-    return {"GB/s": round(2 * slot / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
+    t = [_continuation(run, 100 + i)[0] for i in range(3 * (steps + 2))]
+
+    def timed(kernel, k0):
+        bc.bc_cache_set_kernel(run.h, kernel)
+        for i in range(2):
+            bc.bc_cache_push(run.h, ptrs, t[k0 + i], run.stream)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record()
+        for i in range(steps):
+            bc.bc_cache_push(run.h, ptrs, t[k0 + 2 + i], run.stream)
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / steps
+
+    gbs = lambda ms: round(2 * slot / (ms * 1e-3) / 1e9, 1)
+    by_kernel = {"register": gbs(timed(bc.KERNEL_REGISTER, 0)),
+                 "pipeline": gbs(timed(bc.KERNEL_PIPELINE, steps + 2))}
+    ms = timed(bc.KERNEL_AUTO, 2 * (steps + 2))
+    bc.bc_cache_check(run.h)
+    return {"GB/s": gbs(ms), "ms": round(ms, 4), "GB/s_by_kernel": by_kernel,
             "bytes_per_push": 2 * slot, "pushes": steps,
             "what": "grouped byte-exact copy of one slot (read + write)"}
 

@@ -37,10 +37,10 @@
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
  *    stream (or with the caller's own synchronisation).
  *  - No exception crosses the ABI and device code never traps.  The forecast kernel for
- *    H <= 3 and the large-probe drift kernel wait on their own shared-memory pipelines (TMA
- *    bulk copies completing on mbarriers); every such wait gives up after about one second,
- *    records the failure in the handle's device status word and returns, so the device
- *    never hangs: bc_cache_check reports it.
+ *    H <= 3 and the large drift and push kernels wait on their own shared-memory
+ *    pipelines (TMA bulk copies completing on mbarriers); every such wait gives up after
+ *    about one second, records the failure in the handle's device status word and
+ *    returns, so the device never hangs: bc_cache_check reports it.
  */
 #ifndef BARYCACHE_H
 #define BARYCACHE_H
@@ -107,7 +107,7 @@ typedef struct {
     int64_t kernel_launches; /* CUDA kernels this handle has launched */
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
-    int64_t pipeline_launches; /* of kernel_launches: TMA pipeline kernels (forecast or drift) */
+    int64_t pipeline_launches; /* of kernel_launches: TMA pipeline kernels (any call) */
 } bc_stats;
 
 /* ---------------------------------------------------------------- host-only calls */
@@ -165,7 +165,8 @@ bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
 /* Replace the weight parameters (clears the weight memo). */
 bc_status bc_cache_set_params(bc_handle h, const bc_params *p);
 
-/* Pin the kernel of this handle's forecasts and probe drifts (bc_kernel; default AUTO). */
+/* Pin the kernel of this handle's forecasts, probe drifts and push copies (bc_kernel;
+ * default AUTO). */
 bc_status bc_cache_set_kernel(bc_handle h, int kernel);
 
 /* Forget every pushed node (the arena keeps its bytes; nothing is enqueued). */
@@ -173,10 +174,14 @@ bc_status bc_cache_reset(bc_handle h);
 
 /* Insert a full-step feature (Eq. 6): the oldest slot is evicted by rotating the ring
  * head, and layer_ptrs[l] (device, numels[l] elements of the cache dtype, 16-byte
- * aligned) is copied into it by one grouped copy kernel on `stream`.  `t` is the
- * timestep of this full step.  Errors: INVALID_ARG (null pointer, non-finite t, source
- * overlapping the arena), ALIGNMENT, DUPLICATE_NODE (t equals a node that stays in the
- * window), CUDA. */
+ * aligned) is copied into it by one grouped, byte-exact copy kernel on `stream`: with
+ * AUTO, TMA bulk copies through a three-stage shared-memory ring (one warp per SM) once the
+ * push has at least 16 tiles of 32 KiB per SM, else register loads and stores.  The node
+ * counts as pushed when the call returns; if the pipeline copy gives up waiting (reported
+ * by bc_cache_check) the slot's contents are undefined and the cache should be reset.  `t`
+ * is the timestep of this full step.  Errors: INVALID_ARG (null pointer, non-finite t,
+ * source overlapping the arena), ALIGNMENT, DUPLICATE_NODE (t equals a node that stays in
+ * the window), CUDA. */
 bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, void *stream);
 
 /* Zero-copy push, part 1: the device addresses (one per layer) of the slot the next push
@@ -325,8 +330,8 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
 bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
                                  double *out, void *stream);
 
-/* Report device-side failures of this handle's forecast and drift launches since the last
- * check: BC_ERR_DEVICE_TIMEOUT if any launch gave up waiting for its shared-memory pipeline
+/* Report device-side failures of this handle's forecast, drift and push launches since the
+ * last check: BC_ERR_DEVICE_TIMEOUT if any launch gave up waiting for its shared-memory pipeline
  * (its outputs may then be incomplete), else BC_OK.  Waits for all work on the device, reads and
  * clears the handle's device status word.  Errors: BAD_HANDLE, CUDA, DEVICE_TIMEOUT. */
 bc_status bc_cache_check(bc_handle h);
@@ -336,7 +341,8 @@ bc_status bc_cache_check(bc_handle h);
  * every CTA's pipeline unarmed, so that its bounded wait runs out (about one second) and the
  * launch returns early with the status word set, which bc_cache_check then reports;
  * what = 2 does the same to the next probe drift of at least one 16 KiB tile (its out[]
- * then reads NaN); what = 0 cancels a pending injection.  Nothing is faulted: the copies
+ * then reads NaN); what = 3 to the next push copy (the pushed slot is then undefined);
+ * what = 0 cancels a pending injection.  Nothing is faulted: the copies
  * that were issued complete and are drained. */
 bc_status bc_cache_inject_fault(bc_handle h, int what);
 

@@ -217,7 +217,8 @@ struct bc_cache {
     double *probe_partials = nullptr;             // device scratch of bc_probe_drift
     uint32_t *status = nullptr;                   // device status word of the forecast kernels
     bool inject_next = false;                     // test hooks (bc_cache_inject_fault):
-    bool inject_next_drift = false;               //   next forecast / next probe drift
+    bool inject_next_drift = false;               //   next forecast / probe drift / push
+    bool inject_next_push = false;
     int kernel = BC_KERNEL_AUTO;                  // bc_kernel
 
     char *slot_base(int slot) const { return arena + static_cast<uint64_t>(slot) * slot_bytes; }
@@ -621,8 +622,11 @@ bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, vo
         if (!entries.empty()) {
             DeviceGuard g(h->device);
             if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+            bc::CopyOptions opt{h->kernel, h->status, h->inject_next_push ? 1 : 0};
             const int err = bc::launch_copy(entries.data(), static_cast<int>(entries.size()),
-                                            h->dtype, stream, &h->stats.kernel_launches);
+                                            h->dtype, opt, stream, &h->stats.kernel_launches,
+                                            &h->stats.pipeline_launches);
+            h->inject_next_push = false;
             if (err != cudaSuccess) return cuda_fail(err, "push copy launch");
         }
         rotate_in(h, t);
@@ -938,9 +942,10 @@ bc_status bc_cache_inject_fault(bc_handle h, int what) {
     t_last_error.clear();
     bc_status s = check_handle(h);
     if (s != BC_OK) return s;
-    if (what < 0 || what > 2) return fail(BC_ERR_INVALID_ARG, "unknown fault %d", what);
+    if (what < 0 || what > 3) return fail(BC_ERR_INVALID_ARG, "unknown fault %d", what);
     h->inject_next = (what == 1);
     h->inject_next_drift = (what == 2);
+    h->inject_next_push = (what == 3);
     return BC_OK;
 }
 

@@ -139,8 +139,15 @@ int64_t static_drift_max_elems(bc_dtype dtype);
 int launch_drift_static(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
                         double *out, void *stream, int64_t *launches);
 
-// Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst absolute).
-int launch_copy(const LayerEntry *layers, int n_layers, bc_dtype dtype, void *stream,
-                int64_t *launches);
+// Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst absolute):
+// the TMA bulk-copy pipeline for large pushes (or when pinned / injected), else the
+// register copy.  *pipeline_launches counts the former.
+struct CopyOptions {
+    int kernel;               // bc_kernel
+    uint32_t *status;         // device status word
+    int inject;               // test hook: leave the pipeline's first stage unarmed
+};
+int launch_copy(const LayerEntry *layers, int n_layers, bc_dtype dtype, const CopyOptions &opt,
+                void *stream, int64_t *launches, int64_t *pipeline_launches);
 
 }  // namespace bc

@@ -5,6 +5,7 @@ import pytest
 import torch
 
 from paper_2608_28670_gb300 import barycache as bc
+from tests.gpu_helpers import device_view
 
 pytestmark = pytest.mark.gpu
 
@@ -200,10 +201,35 @@ def test_drift_pipeline_wait_timeout_is_reported_and_recovers():
         bc.bc_cache_destroy(h)
 
 
+def test_push_pipeline_wait_timeout_is_reported_and_recovers():
+    """The push copy's pipeline form under the same test hook: the launch gives up, the
+    check reports it once, and the next push on the handle copies every byte."""
+    import time
+    n = 16384 * 40 + 7
+    src = torch.arange(n, dtype=torch.float32, device="cuda")
+    h = bc.bc_cache_create([n], 2, bc.DTYPE_F32)
+    bc.bc_cache_set_kernel(h, bc.KERNEL_PIPELINE)
+    try:
+        bc.bc_cache_inject_fault(h, 3)
+        t0 = time.perf_counter()
+        bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())
+        assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
+        assert 0.5 < time.perf_counter() - t0 < 60.0
+        bc.bc_cache_check(h)
+        bc.bc_cache_reset(h)
+        bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())
+        bc.bc_cache_check(h)
+        got = device_view(bc.bc_cache_slot_ptrs(h, 0, 1)[0], n, bc.DTYPE_F32)
+        assert torch.equal(got, src)
+        assert bc.bc_cache_stats(h)["pipeline_launches"] == 2
+    finally:
+        bc.bc_cache_destroy(h)
+
+
 def test_check_is_clean_after_normal_launches_and_rejects_unknown_choices():
     h = bc.bc_cache_create([4096], 2, bc.DTYPE_BF16)
     try:
-        assert _status(bc.bc_cache_inject_fault, h, 7) == bc.ERR_INVALID_ARG
+        assert _status(bc.bc_cache_inject_fault, h, 4) == bc.ERR_INVALID_ARG
         assert _status(bc.bc_cache_inject_fault, h, -1) == bc.ERR_INVALID_ARG
         assert _status(bc.bc_cache_set_kernel, h, 3) == bc.ERR_INVALID_ARG
         bc.bc_cache_check(h)

@@ -179,21 +179,41 @@ def test_exact_mode_node_hit_returns_the_node():
         bc.bc_cache_destroy(h)
 
 
-def test_push_copy_is_byte_exact():
-    # Includes NaN payloads and -0.0: the push must move bytes, not values.
-    n = 3 * 8192 + 3
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+@pytest.mark.parametrize("dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+def test_push_copy_is_byte_exact(kernel, dt):
+    # Includes NaN payloads and -0.0: the push must move bytes, not values.  Layer sizes
+    # span whole and ragged 32 KiB pipeline tiles, ends shorter than 16 bytes and a layer
+    # smaller than one 16-byte group.
+    eb = 2 if dt == bc.DTYPE_BF16 else 4
+    numels = [3 * 8192 + 3, 3 * 8192 + 4, 16384 // eb * 5, 3, 100_003]
     rng = np.random.default_rng(1)
-    bits = rng.integers(0, 2 ** 16, n, dtype=np.uint16)
-    bits[:4] = [0x7FC1, 0xFFFF, 0x8000, 0x7F80]
-    h = bc.bc_cache_create([n, n + 1], 2, bc.DTYPE_BF16)
+    src = []
+    for n in numels:
+        if dt == bc.DTYPE_BF16:
+            bits = rng.integers(0, 2 ** 16, n, dtype=np.uint16)
+            bits[:min(n, 4)] = [0x7FC1, 0xFFFF, 0x8000, 0x7F80][:min(n, 4)]
+            src.append(to_device(bits))
+        else:
+            bits = rng.integers(0, 2 ** 32, n, dtype=np.uint64).astype(np.uint32)
+            bits[:min(n, 3)] = [0x7FC00001, 0xFFFFFFFF, 0x80000000][:min(n, 3)]
+            src.append(to_device(bits.view(np.float32)))
+    h = bc.bc_cache_create(numels, 2, dt)
+    bc.bc_cache_set_kernel(h, kernel)
     try:
-        src = [to_device(bits), to_device(np.concatenate([bits, bits[:1]]))]
+        p0 = bc.bc_cache_stats(h)["pipeline_launches"]
         bc.bc_cache_push(h, [s.data_ptr() for s in src], 0.5, stream())
         torch.cuda.synchronize()
-        slots = bc.bc_cache_slot_ptrs(h, 0, 2)
+        bc.bc_cache_check(h)
+        assert bc.bc_cache_stats(h)["pipeline_launches"] - p0 == \
+            (1 if kernel == bc.KERNEL_PIPELINE else 0)
+        slots = bc.bc_cache_slot_ptrs(h, 0, len(numels))
         for l, s in enumerate(src):
-            got = device_view(slots[l], s.numel(), bc.DTYPE_BF16)
-            assert torch.equal(got, s)
+            got = device_view(slots[l], s.numel(), dt)
+            if dt == bc.DTYPE_F32:
+                assert torch.equal(got.view(torch.int32), s.view(torch.int32))
+            else:
+                assert torch.equal(got, s)
     finally:
         bc.bc_cache_destroy(h)
 

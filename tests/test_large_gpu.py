@@ -121,7 +121,7 @@ def test_probe_drift_past_2_pow_31_elements(big):
     assert ei.value.status == bc.ERR_INVALID_ARG
 
 
-def test_push_copy_past_4_gib_is_byte_exact(big):
+def test_push_copy_past_4_gib_is_byte_exact_both_kernels(big):
     h = big
     src = torch.empty(N, dtype=torch.int16, device="cuda")
     synth.fill_device(src.data_ptr(), bc.DTYPE_BF16, N, seed=SEED + 1, tensor_id=0,
@@ -130,11 +130,15 @@ def test_push_copy_past_4_gib_is_byte_exact(big):
     src[N - 1] = -1                              # a NaN payload in the last element
     torch.cuda.synchronize()
     try:
-        bc.bc_cache_push(h, [src.data_ptr()], 0.5, stream())
-        torch.cuda.synchronize()
-        got = device_view(bc.bc_cache_slot_ptrs(h, 0, 1)[0], N, bc.DTYPE_BF16)
-        assert torch.equal(got, src)
-        assert bc.bc_cache_nodes(h) == [0.5, 0.6, 0.65]
+        for kern, t in ((bc.KERNEL_REGISTER, 0.5), (bc.KERNEL_PIPELINE, 0.45)):
+            bc.bc_cache_set_kernel(h, kern)
+            bc.bc_cache_push(h, [src.data_ptr()], t, stream())
+            torch.cuda.synchronize()
+            bc.bc_cache_check(h)
+            got = device_view(bc.bc_cache_slot_ptrs(h, 0, 1)[0], N, bc.DTYPE_BF16)
+            assert torch.equal(got, src)
+        assert bc.bc_cache_nodes(h) == [0.45, 0.5, 0.6]
+        bc.bc_cache_set_kernel(h, bc.KERNEL_AUTO)
     finally:
         del src
         torch.cuda.empty_cache()
