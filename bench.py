@@ -47,6 +47,8 @@ def parse_args():
     ap.add_argument("--e2e-host-cap-gb", type=float, default=48.0,
                     help="page-locked host memory for the e2e leg, shared by the node's ranks")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--probe-elems", type=int, default=None,
+                    help="elements of the probe-drift leg (default: one layer)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -352,7 +354,7 @@ def run_ours(args):
                 result["cpu_baseline"] = cpu_baseline_from_device(run, args.cpu_seconds)
         if not args.no_extra:
             with nvtx_range("probe_drift"):
-                result["probe_drift"] = time_probe(run, args.steps)
+                result["probe_drift"] = time_probe(run, args.steps, args.probe_elems)
             with nvtx_range("push"):
                 result["push"] = time_push(run, args.steps)
     finally:
@@ -428,14 +430,18 @@ def time_push(run, steps):
             "what": "grouped byte-exact copy of one slot (read + write)"}
 
 
-def time_probe(run, steps):
+def time_probe(run, steps, probe_elems=None):
     """Row f3: the probe drift of the adaptive schedule over one cached layer (newest vs the
-    previous node's copy of layer 0): 2 x numel x b bytes, two launches per call."""
+    previous node's copy of layer 0): 2 x numel x b bytes, two launches per call.
+    `probe_elems` probes that many elements from the start of the two slots instead (a
+    flat view across layers; at most one slot)."""
     import torch
     from paper_2608_28670_gb300 import barycache as bc
     if len(run.problem.nodes) < 2:
         return None
     n = run.numels[0]
+    if probe_elems:
+        n = min(int(probe_elems), bc.bc_cache_layout(run.h)[-1] // run.w.elem_bytes)
     cur = bc.bc_cache_slot_ptrs(run.h, 0, len(run.numels))[0]
     prev = bc.bc_cache_slot_ptrs(run.h, 1, len(run.numels))[0]
     out = torch.empty(3, dtype=torch.float64, device="cuda")
@@ -453,7 +459,8 @@ def time_probe(run, steps):
     nbytes = 2 * n * run.w.elem_bytes
     return {"GB/s": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
             "elements": n, "bytes_per_call": nbytes, "drift": round(float(out[2].item()), 6),
-            "what": "bc_probe_drift over layer 0 (newest vs previous node)"}
+            "what": "bc_probe_drift over layer 0 (newest vs previous node)" if not probe_elems
+                    else "bc_probe_drift over the first elements of the two newest slots"}
 
 
 def time_sampling_loop(stream):
