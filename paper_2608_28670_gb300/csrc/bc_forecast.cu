@@ -654,10 +654,15 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
 }
 
 // ------------------------------------------------------------------ launch plumbing
+//
+// The launchers keep a few values computed on first use (SM counts, occupancies, whether a
+// kernel's shared-memory attribute was set on a device).  Handles may be driven from
+// several host threads at once, so these caches are atomics; threads that race to fill
+// one store the same value.
 
 // SM count of the current device, cached per device.
 int sm_count() {
-    static int cached[64] = {};
+    static std::atomic<int> cached[64];
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
     if (dev >= 64) {
@@ -665,28 +670,33 @@ int sm_count() {
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
         return n > 0 ? n : 1;
     }
-    if (cached[dev] == 0) {
+    int c = cached[dev].load(std::memory_order_relaxed);
+    if (c == 0) {
         int n = 0;
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        cached[dev] = n > 0 ? n : 1;
+        c = n > 0 ? n : 1;
+        cached[dev].store(c, std::memory_order_relaxed);
     }
-    return cached[dev];
+    return c;
 }
 
 // Resident CTAs per SM for a kernel, optionally capped (the forecast runs best at two
 // 256-thread CTAs per SM; the single-stream copy at full occupancy).
 template <class KernelPtr>
-int resident_ctas(KernelPtr kern, int &cache, int cap) {
-    if (cache == 0) {
+int resident_ctas(KernelPtr kern, std::atomic<int> &cache, int cap) {
+    int c = cache.load(std::memory_order_relaxed);
+    if (c == 0) {
         int n = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, kThreads, 0) != cudaSuccess ||
             n < 1)
             n = 1;
         if (cap > 0 && cap < n) n = cap;
-        cache = n;
+        c = n;
+        cache.store(c, std::memory_order_relaxed);
     }
-    return cache;
+    return c;
 }
+
 
 template <int CAP>
 int64_t fill_table(ForecastArgs<CAP> &a, const LayerEntry *layers, int n, int elem_bytes,
@@ -734,15 +744,9 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         // shared-memory pipeline, one CTA per SM
         auto kern = forecast_tma_kernel<K, TIn, TOut, CAP>;
         constexpr int smem = kTmaSmemBytes<K>;
-        static bool attr_set[64] = {};  // the attribute is per device
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev < 0 || dev >= 64 || !attr_set[dev]) {
-            const int err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 smem);
-            if (err != cudaSuccess) return err;
-            if (dev >= 0 && dev < 64) attr_set[dev] = true;
-        }
+        static std::atomic<bool> attr_set[64];
+        const int err = ensure_smem_attribute(kern, attr_set, smem);
+        if (err != cudaSuccess) return err;
         const int64_t cap = sm_count();
         const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
         kern<<<grid, kThreads, smem, s>>>(a);
@@ -751,7 +755,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         return cudaGetLastError();
       }
     }
-    static int occ = 0;
+    static std::atomic<int> occ{0};
     auto kern = forecast_kernel<K, TIn, TOut, CAP>;
     const int64_t cap =
         static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ, BC_CTAS_PER_SM);
@@ -793,7 +797,7 @@ int dispatch_dtypes(const LaunchPlan &p, cudaStream_t s, int64_t *launches, int6
 template <class T, int CAP>
 int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStream_t s,
                int64_t *launches, int64_t *pipeline_launches) {
-    static int occ = 0;
+    static std::atomic<int> occ{0};
     ForecastArgs<CAP> a;
     memset(&a, 0, sizeof a);
     a.euler_layer = -1;
@@ -808,15 +812,9 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
          a.total_tiles >= static_cast<int64_t>(kCopyMinTilesPerCta) * sm_count());
     if (pipeline) {
         auto kern = copy_tma_kernel<T, CAP>;
-        static bool attr_set[64] = {};  // the attribute is per device
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev < 0 || dev >= 64 || !attr_set[dev]) {
-            const int err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 kCopySmemBytes);
-            if (err != cudaSuccess) return err;
-            if (dev >= 0 && dev < 64) attr_set[dev] = true;
-        }
+        static std::atomic<bool> attr_set[64];
+        const int err = ensure_smem_attribute(kern, attr_set, kCopySmemBytes);
+        if (err != cudaSuccess) return err;
         const int64_t cap = static_cast<int64_t>(sm_count()) * BC_COPY_CTAS_PER_SM;
         const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
         kern<<<grid, kCopyTmaThreads, kCopySmemBytes, s>>>(a);

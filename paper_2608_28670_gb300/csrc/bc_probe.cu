@@ -308,15 +308,9 @@ int launch_drift_tma(const char *cur, const char *prev, int64_t n, int64_t ntile
                      double *partials, int max_parts, const DriftOptions &opt, cudaStream_t s,
                      int *grid_out) {
     auto kern = drift_tma_partials<kBf16>;
-    static bool attr_set[64] = {};  // the attribute is per device
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
-        const int err =
-            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kDriftSmemBytes);
-        if (err != cudaSuccess) return err;
-        if (dev >= 0 && dev < 64) attr_set[dev] = true;
-    }
+    static std::atomic<bool> attr_set[64];
+    const int err = ensure_smem_attribute(kern, attr_set, kDriftSmemBytes);
+    if (err != cudaSuccess) return err;
     int64_t grid = sm_count_of_current_device();
     if (grid > max_parts) grid = max_parts;
     if (grid > ntiles) grid = ntiles;

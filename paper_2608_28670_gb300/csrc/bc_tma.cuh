@@ -10,6 +10,9 @@
 // never in a hung device.
 #pragma once
 
+#include <cuda_runtime.h>
+
+#include <atomic>
 #include <cstdint>
 
 namespace bc {
@@ -101,6 +104,19 @@ __device__ __forceinline__ void bulk_wait_group_read() {
 // Wait until every bulk group of this thread has completed (its writes are performed).
 __device__ __forceinline__ void bulk_wait_group_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// Host side: raise a pipeline kernel's dynamic shared-memory limit to `bytes`, once per
+// device (host threads may race here; they set the same value).
+template <class KernelPtr>
+int ensure_smem_attribute(KernelPtr kern, std::atomic<bool> (&done)[64], int bytes) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && done[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    const int err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (err != cudaSuccess) return err;
+    if (dev >= 0 && dev < 64) done[dev].store(true, std::memory_order_release);
+    return cudaSuccess;
 }
 
 }  // namespace bc
