@@ -4,7 +4,8 @@
  *   abi_client host     host-only calls (weights, footprints, schedules, errors): no GPU
  *   abi_client device   one cache on the current GPU: allocate with cudaMalloc, push three
  *                       full-step features, forecast, read back, and compare every element
- *                       with the fp64 oracle (liboracle, linked for the check only)
+ *                       with the fp64 oracle (liboracle, linked for the check only); then
+ *                       the probe drift of the two newest slots against the oracle's
  *
  * Exit status 0 on success; a failing check prints what failed and exits 1.
  */
@@ -21,6 +22,7 @@ int oracle_paper_weights(const double *s, int m, double t, double delta, double 
                          double eta, double *W);
 void oracle_combine(int dtype, const void *const *F, int m, const double *W, int64_t n,
                     double *out, double *bound);
+void oracle_drift(int dtype, const void *cur, const void *prev, int64_t n, double *out);
 
 /* The few CUDA runtime calls the device check needs, declared here so that the client
  * compiles with a plain C compiler against libcudart. */
@@ -135,6 +137,21 @@ static int device_checks(void) {
     }
     CHECK(bad == 0, "%lld of %lld elements outside 2^-8 * sum |W||F|", (long long)bad,
           (long long)n);
+    /* probe drift between the two newest slots (device) and the same arrays (oracle) */
+    void *s0[1], *s1[1];
+    double *dev_drift = NULL, drift[3], ref_drift[3];
+    CHECK(bc_cache_slot_ptrs(h, 0, s0) == BC_OK && bc_cache_slot_ptrs(h, 1, s1) == BC_OK,
+          "slot pointers");
+    CHECK(cudaMalloc((void **)&dev_drift, sizeof drift) == 0, "cudaMalloc drift");
+    CHECK(bc_probe_drift(h, s0[0], s1[0], n, BC_DTYPE_BF16, dev_drift, NULL) == BC_OK,
+          "probe drift: %s", bc_last_error());
+    CHECK(cudaMemcpy(drift, dev_drift, sizeof drift, D2H) == 0, "download drift");
+    CHECK(bc_cache_check(h) == BC_OK, "device status after the drift");
+    oracle_drift(1, host[2], host[1], n, ref_drift);
+    for (int i = 0; i < 3; ++i)
+        CHECK(fabs(drift[i] - ref_drift[i]) <= 2e-6 * fabs(ref_drift[i]),
+              "drift[%d] = %.17g, oracle %.17g", i, drift[i], ref_drift[i]);
+    cudaFree(dev_drift);
     bc_stats st;
     CHECK(bc_cache_stats(h, &st) == BC_OK && st.forecasts == 1 && st.pushes == 3, "stats");
     bc_cache_destroy(h);
