@@ -453,7 +453,10 @@ int static_scratch(double **out) {
     if (!g_static_scratch[dev]) {
         void *p = nullptr;
         err = cudaGetSymbolAddress(&p, g_drift_scratch);
-        if (err != cudaSuccess) return err;
+        if (err != cudaSuccess) {
+            cudaGetLastError();  // reported once, by return value
+            return err;
+        }
         g_static_scratch[dev] = static_cast<double *>(p);
     }
     *out = g_static_scratch[dev];

@@ -114,7 +114,10 @@ int ensure_smem_attribute(KernelPtr kern, std::atomic<bool> (&done)[64], int byt
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && done[dev].load(std::memory_order_acquire)) return cudaSuccess;
     const int err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (err != cudaSuccess) return err;
+    if (err != cudaSuccess) {
+        cudaGetLastError();  // reported once, by return value, not again to later calls
+        return err;
+    }
     if (dev >= 0 && dev < 64) done[dev].store(true, std::memory_order_release);
     return cudaSuccess;
 }
