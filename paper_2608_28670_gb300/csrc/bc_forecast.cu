@@ -24,6 +24,10 @@
 // these numbers came from sweeps of vector width, vectors per thread, CTA size and count,
 // cache hints, tile order, ring depth and store path on that workload.
 //
+// The file also holds the push's grouped byte-exact copy on the same layer tables:
+// copy_tma_kernel (TMA bulk loads and stores through a three-stage ring, one warp per SM;
+// large pushes) and copy_kernel (16-byte register copies; small pushes).
+//
 // Outputs, the sampler state and push sources carry only the ABI's 16-byte alignment and
 // use 128-bit (or 64-bit) accesses; stores are st.global.cs (streaming).  No CTA waits on
 // another, nothing allocates and nothing traps: every vector index is checked against its
