@@ -110,7 +110,8 @@ def profiled_traffic(workload: str, K: int):
 
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) during the timed region."""
+    """nvidia-smi samples every 100 ms, started before the warm-up (the tool takes a moment
+    to start); stop(window) keeps the samples whose timestamps fall in the timed region."""
 
     def __init__(self, enabled: bool):
         self.proc = None
@@ -119,7 +120,7 @@ class ClockSampler:
             return
         fd, self.path = tempfile.mkstemp(suffix=".csv")
         os.close(fd)
-        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+        q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
              "clocks_event_reasons.sw_power_cap")
         try:
@@ -130,11 +131,13 @@ class ClockSampler:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", idx, f"--query-gpu={q}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+                 "-lms", "100"], stdout=self.fh, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
 
-    def stop(self):
+    def stop(self, window=None):
+        """Summary of the samples; `window` = (start, end) in time.time() seconds."""
+        import datetime
         if not self.proc:
             return None
         self.proc.terminate()
@@ -143,25 +146,33 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
         self.fh.close()
-        rows = []
+        rows, stamps = [], []
         with open(self.path) as fh:
             for line in fh:
                 f = [x.strip() for x in line.split(",")]
-                if len(f) >= 7:
+                if len(f) >= 8:
                     try:
-                        rows.append((float(f[0]), float(f[1]), float(f[2]), f[3:7]))
+                        rows.append((float(f[1]), float(f[2]), float(f[3]), f[4:8]))
+                        stamps.append(datetime.datetime.strptime(
+                            f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp())
                     except ValueError:
                         pass
         os.unlink(self.path)
         if not rows:
             return None
+        in_window = False
+        if window is not None and len(stamps) == len(rows):
+            kept = [r for r, t in zip(rows, stamps) if window[0] - 0.05 <= t <= window[1] + 0.05]
+            if kept:
+                rows, in_window = kept, True
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i, v in enumerate(r[3]) if v == "Active"})
         loaded = [r for r in rows if r[2] > 300.0] or rows
         return {"sm_mhz": statistics.median(r[0] for r in loaded),
                 "sm_max_mhz": max(r[1] for r in rows),
                 "reasons": reasons, "samples": len(rows), "samples_under_load": len(loaded),
-                "power_w_max": max(r[2] for r in rows)}
+                "power_w_max": max(r[2] for r in rows),
+                "samples_from": "timed region" if in_window else "warm-up and timed region"}
 
 
 class nvtx_range:
@@ -224,6 +235,7 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     host_s = []
     torch.cuda.synchronize()
+    wall0 = time.time()
     with nvtx_range(f"timed {steps} skipped steps"):
         for i in range(steps):
             starts[i].record()
@@ -238,6 +250,7 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     per_step = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     st1 = run.stats()
     launches = st1["kernel_launches"] - launches0
+    time_forecast.window = (wall0, time.time())
     time_forecast.host_us = 1e6 * statistics.median(host_s)
     time_forecast.pipeline = st1["pipeline_launches"] - st0["pipeline_launches"]
     return total_ms, per_step, launches
@@ -272,7 +285,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         clocks = ClockSampler(not args.no_clocks)
         total_ms, per_step, launches = time_forecast(run, args.steps, args.warmup, stream, dist)
-        clk = clocks.stop()
+        clk = clocks.stop(time_forecast.window)
         ms = max_over_ranks(total_ms / args.steps, dist)
         alg = run.algorithmic_bytes()
         value = job_throughput(alg, ms, world)
