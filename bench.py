@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip timing the workload's other history depths K")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-chunk-layers", type=int, default=6,
+                    help="layers per pipelined chunk of the end-to-end leg")
     ap.add_argument("--e2e-host-cap-gb", type=float, default=48.0,
                     help="page-locked host memory for the e2e leg, shared by the node's ranks")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -361,6 +363,7 @@ def run_ours(args):
         if not args.no_e2e:      # before the CPU leg, which loads the host memory system
             with nvtx_range("e2e"):
                 result["e2e"] = e2e(run, args.e2e_steps, world, dist,
+                                    chunk_layers=args.e2e_chunk_layers,
                                     host_cap_bytes=args.e2e_host_cap_gb * 1e9)
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
             with nvtx_range("cpu_baseline"):
