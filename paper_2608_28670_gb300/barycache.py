@@ -122,6 +122,8 @@ def exported_names() -> list[str]:
 def lib() -> ctypes.CDLL:
     """Load the library (raises if it has not been built; there is no fallback)."""
     global _lib
+    if _lib is not None:          # loaded: no lock on the per-call path
+        return _lib
     with _lock:
         if _lib is None:
             if not os.path.exists(LIB_PATH):
