@@ -26,8 +26,10 @@
  *
  * Pins (tests/test_oracle_pins.py, tests/test_oracle_samplers.py): every function is checked
  * against closed forms, identities or library routines.  For the paper's weights with a decay
- * power delta != 1 the paper fixes no value: those are pinned by invariants and limits only
- * (scale invariance, the delta -> 0 limit, sign alternation, unit sum, translation invariance).
+ * power delta != 1 the paper prints no value; they are pinned by hand-derived closed forms at
+ * delta = 2 and 1/2 (where the powers are exact: squares and square roots, including a case
+ * with the clip active) and by invariants and limits (scale invariance, the delta -> 0 limit,
+ * sign alternation, unit sum, translation invariance).
  */
 #include <math.h>
 #include <stdint.h>

@@ -32,6 +32,18 @@ MUTANTS = {
     # Eq. 11: power on the wrong quantity (eta outside, delta ignored)
     "eq11_power_ignored": ("a[j] = sgn_plus(ut[j]) * pow(fabs(ut[j]) + eta, delta);",
                            "a[j] = sgn_plus(ut[j]) * (fabs(ut[j]) + eta);"),
+    # Eqs. 10-11 in the wrong order: the power applied first and its result clipped
+    "eq10_after_eq11": ("    for (int j = 0; j < m; ++j) ut[j] = fmax(-C, fmin(C, u[j]));\n\n"
+                        "    /* Eq. 11 */\n    double sum = 0.0, sum_abs = 0.0;\n"
+                        "    for (int j = 0; j < m; ++j) {\n"
+                        "        a[j] = sgn_plus(ut[j]) * pow(fabs(ut[j]) + eta, delta);",
+                        "    for (int j = 0; j < m; ++j) ut[j] = u[j];\n\n"
+                        "    /* Eq. 11 */\n    double sum = 0.0, sum_abs = 0.0;\n"
+                        "    for (int j = 0; j < m; ++j) {\n"
+                        "        a[j] = fmax(-C, fmin(C, sgn_plus(ut[j]) * pow(fabs(ut[j]) + eta, delta)));"),
+    # Eq. 11: the decay power inverted
+    "eq11_power_inverted": ("a[j] = sgn_plus(ut[j]) * pow(fabs(ut[j]) + eta, delta);",
+                            "a[j] = sgn_plus(ut[j]) * pow(fabs(ut[j]) + eta, 1.0 / delta);"),
     # Eq. 12 as printed: the last weight scaled by lambda instead of a blend towards x_{f=-1}
     "eq12_printed_vector": ("W[j] = (1.0 - lambda) * alpha + (j == 0 ? lambda : 0.0);",
                             "W[j] = (j < m - 1 ? (1.0 - lambda) : lambda) * alpha;"),
