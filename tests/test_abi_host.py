@@ -291,3 +291,20 @@ def test_pointer_tables_from_lists_and_numpy_arrays():
         bc._ptr_array(np.array([16, 32], dtype=np.uint32))
     with pytest.raises(TypeError):
         bc._ptr_array(np.zeros((2, 2), dtype=np.uint64))
+
+
+def _golden():
+    from tests.test_oracle_pins import _golden_rows
+    return _golden_rows()
+
+
+@pytest.mark.parametrize("row", _golden(), ids=lambda r: r["name"])
+def test_library_solver_matches_the_hand_derived_weights(row):
+    # The library's own fp64 solver (not just the oracle) against the worked examples.
+    if row["mode"] == "exact":
+        prm = bc.make_params(mode=bc.MODE_EXACT)
+    else:
+        prm = bc.make_params(mode=bc.MODE_PAPER, delta=row["delta"], lam=row["lam"],
+                             clip_C=row["C"], eta=row["eta"])
+    got = bc.bc_solve(row["nodes"], row["t"], prm)
+    np.testing.assert_allclose(got, row["W"], rtol=1e-12, atol=1e-12)
