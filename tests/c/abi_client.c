@@ -2,6 +2,8 @@
  * abi_client.c -- a plain C client of libbarycache.so, with no Python in between.
  *
  *   abi_client host     host-only calls (weights, footprints, schedules, errors): no GPU
+ *   abi_client hostcost host time of bc_forecast calls on small caches of 1-64 layers
+ *                       (launch included; the GPU work is tiny), one JSON line per size
  *   abi_client device   one cache on the current GPU: allocate with cudaMalloc, push three
  *                       full-step features, forecast, read back, and compare every element
  *                       with the fp64 oracle (liboracle, linked for the check only); then
@@ -9,11 +11,13 @@
  *
  * Exit status 0 on success; a failing check prints what failed and exits 1.
  */
+#define _POSIX_C_SOURCE 199309L
 #include <math.h>
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
+#include <time.h>
 
 #include "barycache.h"
 
@@ -164,11 +168,62 @@ static int device_checks(void) {
     return failures;
 }
 
+static double now_s(void) {
+    struct timespec ts;
+    clock_gettime(CLOCK_MONOTONIC, &ts);
+    return (double)ts.tv_sec + 1e-9 * (double)ts.tv_nsec;
+}
+
+/* Host cost of one forecast call through the ABI (memo hit, table build, launch), on
+ * caches of 1, 4, 16 and 64 layers of 4096 bf16 elements, and of one memo lookup. */
+static int host_cost(void) {
+    enum { kMaxLayers = 64, kCalls = 500, kElems = 4096 };
+    void *src = NULL, *out = NULL;
+    CHECK(cudaMalloc(&src, kElems * 2) == 0 && cudaMalloc(&out, (size_t)kMaxLayers * kElems * 2) == 0,
+          "cudaMalloc");
+    for (int L = 1; L <= kMaxLayers && !failures; L *= 4) {
+        int64_t numels[kMaxLayers];
+        const void *ptrs[kMaxLayers];
+        void *outs[kMaxLayers];
+        for (int l = 0; l < L; ++l) {
+            numels[l] = kElems;
+            ptrs[l] = src;
+            outs[l] = (char *)out + (size_t)l * kElems * 2;
+        }
+        bc_handle h = NULL;
+        CHECK(bc_cache_create(numels, L, 3, BC_DTYPE_BF16, NULL, &h) == BC_OK, "create");
+        const double ts[3] = {0.9, 0.85, 0.8};
+        for (int k = 0; k < 3; ++k) CHECK(bc_cache_push(h, ptrs, ts[k], NULL) == BC_OK, "push");
+        for (int i = 0; i < 100; ++i) bc_forecast(h, 0.75, outs, BC_DTYPE_BF16, NULL);
+        cudaDeviceSynchronize();
+        const double t0 = now_s();
+        for (int i = 0; i < kCalls; ++i)
+            CHECK(bc_forecast(h, 0.75, outs, BC_DTYPE_BF16, NULL) == BC_OK, "forecast");
+        const double t1 = now_s();
+        cudaDeviceSynchronize();
+        const double t2 = now_s();
+        double c[BC_MAX_K];
+        int m = 0;
+        const double t3 = now_s();
+        for (int i = 0; i < kCalls; ++i) bc_coefficients(h, 0.75, c, &m);
+        const double t4 = now_s();
+        CHECK(bc_cache_check(h) == BC_OK, "device status");
+        printf("{\"layers\": %d, \"host_us_per_forecast\": %.2f, \"device_us_per_forecast\": %.2f, "
+               "\"memo_lookup_us\": %.3f}\n", L, 1e6 * (t1 - t0) / kCalls,
+               1e6 * (t2 - t0) / kCalls, 1e6 * (t4 - t3) / kCalls);
+        bc_cache_destroy(h);
+    }
+    cudaFree(src);
+    cudaFree(out);
+    return failures;
+}
+
 int main(int argc, char **argv) {
     if (argc < 2) return 2;
     int rc = 0;
     if (strcmp(argv[1], "host") == 0) rc = host_checks();
     else if (strcmp(argv[1], "device") == 0) rc = device_checks();
+    else if (strcmp(argv[1], "hostcost") == 0) rc = host_cost();
     else return 2;
     printf("%s checks: %s\n", argv[1], rc ? "FAILED" : "ok");
     return rc ? 1 : 0;

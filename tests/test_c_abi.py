@@ -36,3 +36,15 @@ def test_c_client_host_calls(client):
 def test_c_client_full_forecast_on_the_device(client):
     p = subprocess.run([client, "device"], capture_output=True, text=True, timeout=300)
     assert p.returncode == 0, p.stdout + p.stderr
+
+
+@pytest.mark.gpu
+def test_c_client_host_cost_mode_runs(client):
+    # The timing mode reports one JSON line per cache size; the numbers are measurements,
+    # so only their presence and sanity are checked here.
+    import json
+    p = subprocess.run([client, "hostcost"], capture_output=True, text=True, timeout=300)
+    assert p.returncode == 0, p.stdout + p.stderr
+    rows = [json.loads(l) for l in p.stdout.splitlines() if l.startswith("{")]
+    assert [r["layers"] for r in rows] == [1, 4, 16, 64]
+    assert all(0 < r["host_us_per_forecast"] < 1000 and r["memo_lookup_us"] > 0 for r in rows)
