@@ -210,9 +210,10 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  *     out_l[e] = sum_{j=1..m} W_j * F_{l,j}[e],   m = min(pushed, K),
  * with W from the solver (memoised by Diff Key, rounded to fp32), fp32 accumulation in
  * node order j = 1..m, and the result stored as `out_dtype` (bf16: round to nearest even).
- * One persistent grouped kernel launch covers every selected layer (more only for
- * caches of several hundred layers).  Layers with a NULL output are skipped, which also
- * serves to forecast a window of layers.  Outputs must not overlap the arena.
+ * One persistent grouped kernel launch covers every selected layer (one per 1016 layers
+ * beyond that).  Layers with a NULL output are skipped, which also serves to forecast a
+ * window of layers.  Outputs must not overlap the arena (checked) or each other (not
+ * checked: overlapping outputs race).
  * Errors: INVALID_ARG, ALIGNMENT, NOT_READY, DEGENERATE_WEIGHTS, CUDA. */
 bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
                       void *stream);
