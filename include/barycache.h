@@ -90,16 +90,19 @@ typedef struct {
 
 typedef struct bc_cache *bc_handle;
 
-/* Kernel selection (bc_cache_set_kernel), for forecasts and the probe drift.  Forecasts,
- * AUTO: the shared-memory pipeline (TMA bulk copies into a three-stage ring, one CTA per SM)
- * for H <= 3 when the launch has at least 16 tiles of 8 Ki bf16 / 4 Ki fp32 elements per SM,
- * else the register kernel (each thread holds its history loads in registers; up to two
- * CTAs per SM); H = 4 launches always use the register kernel; both compute the same
- * bits.  Probe
- * drift, AUTO: the pipeline form (a five-stage ring of 16 KiB tiles of both tensors, one
- * CTA per SM) from 16 such tiles per SM on, else register loads; the two forms group the
- * partial sums differently, so they agree within rounding, not bit for bit.  REGISTER /
- * PIPELINE pin one. */
+/* Kernel selection (bc_cache_set_kernel) for forecasts, probe drifts and push copies.
+ * AUTO picks per launch:
+ *  - forecast: the shared-memory pipeline (TMA bulk copies into a three-stage ring, one CTA
+ *    per SM) for H <= 3 when the launch has at least 16 tiles of 8 Ki bf16 / 4 Ki fp32
+ *    elements per SM, else the register kernel (each thread holds its history loads in
+ *    registers; up to two CTAs per SM); H = 4 always uses the register kernel.  Both
+ *    compute the same bits.
+ *  - probe drift: the pipeline form (a five-stage ring of 16 KiB tiles of both tensors, one
+ *    CTA per SM) from 16 such tiles per SM on, else register loads.  The two forms group
+ *    the partial sums differently, so they agree within rounding, not bit for bit.
+ *  - push copy: TMA bulk loads and stores through a three-stage ring (one warp per SM) from
+ *    16 tiles of 32 KiB per SM on, else register copies.  Both are byte-exact.
+ * REGISTER / PIPELINE pin one form for all three. */
 typedef enum { BC_KERNEL_AUTO = 0, BC_KERNEL_REGISTER = 1, BC_KERNEL_PIPELINE = 2 } bc_kernel;
 
 typedef struct {
