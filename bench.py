@@ -4,14 +4,20 @@
 One step = one skipped diffusion step of the workload: the host weight solve (Diff Key memo,
 Eqs. 8-12) plus the grouped forecast kernel over every cached layer (Eq. 13), issued through
 the C ABI on a torch stream.  Inputs (the K history slots) are resident in HBM before the
-timed region and are far larger than L2 (so no L2 flush is needed).  Steps alternate between
-the skipped steps that share one history window, as in the equal-spaced schedule.
+timed region; they are far larger than L2 except for c2i-256, where L2 is flushed before
+every step outside its events.  Steps alternate between the skipped steps that share one
+history window, as in the equal-spaced schedule.
 
 Prints one JSON line (rank 0).  Default workload: the video DiT (60 x [1, 118800, 3072] bf16,
-K = 3; 131 GB of cache, 175 GB of HBM traffic per step).
+K = 3; 131 GB of cache, 175 GB of HBM traffic per step).  Beside the headline the line
+carries the roofline of the dominant kernel, the K sweep, the end-to-end leg with host
+buffers, the oracle on the host cores, and the legs of the other rows (push, probe drift,
+fused step, sampling loop, graph-captured loop, blockwise cache, other workloads).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload t2v|mmdit-t2i|t2i-1024|c2i-512|c2i-256] [--K 3] [--no-sweep]
+                    [--no-e2e] [--no-cpu-baseline] [--no-clocks] [--no-extra]
+                    [--e2e-steps S] [--e2e-chunk-layers C] [--probe-elems N]
 """
 from __future__ import annotations
 
