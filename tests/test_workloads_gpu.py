@@ -41,10 +41,10 @@ def gather(ptr: int, n: int, dtype: int, idx: torch.Tensor) -> np.ndarray:
     return a.view(np.uint16) if dtype == bc.DTYPE_BF16 else a
 
 
-def check_run(run: WorkloadRun, rng, calls=None, full=lambda l: True):
+def check_run(run: WorkloadRun, rng, calls=None, full=lambda l: True, mode=bc.MODE_PAPER):
     w, h = run.w, run.h
     p = run.problem
-    W = oracle_weights(list(p.nodes), p.t, bc.MODE_PAPER)
+    W = oracle_weights(list(p.nodes), p.t, mode)
     assert bc.bc_cache_nodes(h) == list(p.nodes)
     m = len(p.nodes)
     slot_ptrs = [bc.bc_cache_slot_ptrs(h, j, len(run.numels)) for j in range(m)]
@@ -112,6 +112,22 @@ def test_image_workloads_every_element(name):
         check_run(run, np.random.default_rng(len(name)))
         st = run.stats()
         assert st["kernel_launches"] == 1 and st["forecasts"] == 1
+    finally:
+        run.close()
+        torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name,out_dtype,mode", [
+    ("mmdit-t2i", bc.DTYPE_F32, bc.MODE_PAPER),     # fp32 outputs beside the fused Euler step
+    ("c2i-512", bc.DTYPE_BF16, bc.MODE_EXACT),      # exact barycentric weights, H = 4
+    ("t2i-1024", bc.DTYPE_F32, bc.MODE_EXACT),
+], ids=["mmdit-f32-paper", "c2i512-bf16-exact", "t2i-f32-exact"])
+def test_image_workloads_other_weights_and_output_dtypes(name, out_dtype, mode):
+    torch.cuda.empty_cache()
+    run = WorkloadRun(WORKLOADS[name], out_dtype=out_dtype, params=bc.make_params(mode=mode),
+                      stream=stream())
+    try:
+        check_run(run, np.random.default_rng(7), mode=mode)
     finally:
         run.close()
         torch.cuda.empty_cache()
