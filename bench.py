@@ -1085,7 +1085,8 @@ def cpu_baseline_from_device(run, seconds):
         pool.close()
     return {"value": round(elems * per_elem / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
             "kind": "oracle", "elems_per_s": round(elems / secs, 1),
-            "sample": f"{sample[0].size} elements (64 chunks of {CHUNK} consecutive elements, "
+            "sample": f"{sample[0].size} elements ({n_chunks} chunks of "
+                      f"{max(x.size for x in parts[0])} consecutive elements, "
                       f"layers round-robin) of the K={m} history slots, processed {1 + passes} "
                       f"times by {cores} spawned workers running the fp64 oracle, {secs:.1f} s",
             "single_core": {"value": round(n1 * per_elem / t1 / 1e9, 4), "cores": 1,
