@@ -26,9 +26,10 @@
  *    device work is enqueued on it asynchronously; errors are reported by return value
  *    only, and no call blocks on the device except bc_cache_create/destroy and
  *    bc_cache_check.
- *  - CUDA graphs: pushes, commits, forecasts (all variants) and the probe drift enqueue
- *    kernels only (no allocation, copy or synchronisation), so they may be called while
- *    `stream` is being captured.  The graph holds the slot addresses, weights and update
+ *  - CUDA graphs: while `stream` is being captured, pushes, commits, forecasts (all
+ *    variants) and the probe drift enqueue kernels only (no allocation, copy or
+ *    synchronisation), so they may be called during capture (outside capture, a forecast
+ *    over more than 1016 layers may also copy its layer table to the device).  The graph holds the slot addresses, weights and update
  *    coefficients chosen when each call was made; replaying it repeats that device work
  *    and does not move the handle's host state (ring head, node times, statistics).  The
  *    first forecast of each kind on a device also queries and sets per-device kernel
@@ -36,8 +37,8 @@
  *  - Host-side cache state (ring head, node times) changes when the call is made, so
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
  *    stream (or with the caller's own synchronisation).
- *  - No exception crosses the ABI and device code never traps.  The forecast kernel for
- *    H <= 3 and the large drift and push kernels wait on their own shared-memory
+ *  - No exception crosses the ABI and device code never traps.  The pipeline forecast
+ *    kernel and the large drift and push kernels wait on their own shared-memory
  *    pipelines (TMA bulk copies completing on mbarriers); every such wait gives up after
  *    about one second, records the failure in the handle's device status word and
  *    returns, so the device never hangs: bc_cache_check reports it.
@@ -95,7 +96,8 @@ typedef struct bc_cache *bc_handle;
  *  - forecast: the shared-memory pipeline (TMA bulk copies into a three-stage ring, one CTA
  *    per SM) for H <= 3 when the launch has at least 16 tiles of 8 Ki bf16 / 4 Ki fp32
  *    elements per SM, else the register kernel (each thread holds its history loads in
- *    registers; up to two CTAs per SM); H = 4 always uses the register kernel.  Both
+ *    registers; up to two CTAs per SM; half-size tiles when the launch has fewer than two
+ *    tiles per SM); H = 4 uses the register kernel unless PIPELINE is pinned.  All forms
  *    compute the same bits.
  *  - probe drift: the pipeline form (a five-stage ring of 16 KiB tiles of both tensors, one
  *    CTA per SM) from 16 such tiles per SM on, else register loads.  The two forms group
@@ -112,6 +114,7 @@ typedef struct {
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
     int64_t pipeline_launches; /* of kernel_launches: TMA pipeline kernels (any call) */
+    int64_t table_uploads;   /* device layer-table uploads (forecasts of > 1016 layers) */
 } bc_stats;
 
 /* ---------------------------------------------------------------- host-only calls */
@@ -148,9 +151,10 @@ bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtyp
 /* Create the cache context H_t of Eq. 6 for `n_layers` tensors of numels[l] elements of
  * `dtype`, with history length K (1..BC_MAX_K).  Allocates, on the current device, one
  * arena of bc_cache_bytes_for(...) bytes and 16 KiB of reduction scratch for
- * bc_probe_drift plus a status word (the only device allocations the library makes; freed
- * by bc_cache_destroy).  p == NULL uses the paper's defaults.  Blocks until the allocation is
- * done.  Errors: INVALID_ARG, OOM, CUDA. */
+ * bc_probe_drift plus a status word, and for caches of more than 1016 layers a layer table
+ * of 32 bytes per layer in device memory and the same in pinned host memory (the only
+ * allocations the library makes; freed by bc_cache_destroy).  p == NULL uses the paper's
+ * defaults.  Blocks until the allocation is done.  Errors: INVALID_ARG, OOM, CUDA. */
 bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
                           const bc_params *p, bc_handle *out);
 
@@ -214,10 +218,18 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  *     out_l[e] = sum_{j=1..m} W_j * F_{l,j}[e],   m = min(pushed, K),
  * with W from the solver (memoised by Diff Key, rounded to fp32), fp32 accumulation in
  * node order j = 1..m, and the result stored as `out_dtype` (bf16: round to nearest even).
- * One persistent grouped kernel launch covers every selected layer (one per 1016 layers
- * beyond that).  Layers with a NULL output are skipped, which also serves to forecast a
- * window of layers.  Outputs must not overlap the arena (checked) or each other (not
- * checked: overlapping outputs race).
+ * The fp32 weights are divided by a power of two s >= sum_j |W_j| and the sum multiplied by s
+ * at the end: the same bits wherever the plain fp32 sum neither overflows nor goes
+ * subnormal, and finite inputs never overflow in a partial sum.  NaN and +-Inf in the history
+ * propagate by IEEE rules (a NaN stays NaN; W_j * Inf is an infinity of W_j's sign).
+ * One persistent grouped kernel launch covers every selected layer.  Beyond 1016 selected
+ * layers the launch reads its layer table from the handle's device copy, which is
+ * re-uploaded (one cudaMemcpyAsync on `stream`, from pinned memory) only when the outputs
+ * differ from the previous such call; while `stream` is being captured into a CUDA graph it
+ * issues one launch per 1016 layers instead, so that the graph holds its own tables.
+ * Layers with a NULL output are skipped, which also serves to forecast a window of layers.
+ * Outputs must not overlap the arena (checked) or each other (not checked: overlapping
+ * outputs race).
  * Errors: INVALID_ARG, ALIGNMENT, NOT_READY, DEGENERATE_WEIGHTS, CUDA. */
 bc_status bc_forecast(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
                       void *stream);
@@ -236,7 +248,9 @@ bc_status bc_forecast_step(bc_handle h, double t_new, double dt, void *const *ou
 /* Forecast fused with a general sampler update on layer `v_layer` (the cached model output,
  * e.g. the noise prediction eps of Eq. 3 or a flow velocity), in the same launch as the
  * forecast of every other selected layer:
- *     v_hat[e] = sum_j W_j V_j[e],    x[e] <- a x[e] + b v_hat[e] + c z[e]   (fp32 math)
+ *     v_hat[e] = sum_j W_j V_j[e],    x[e] <- a x[e] + b v_hat[e] + c z[e]   (fp32 math;
+ * b v_hat is formed inside one FMA from the scaled sum, so x stays finite where only v_hat
+ * itself would exceed the fp32 range)
  * z (device, numels[v_layer] elements of x_dtype, 16-byte aligned, read only) may be NULL
  * (no noise term).  Coefficients for the DDPM mean of Eq. 3 and for DDIM come from
  * bc_ddpm_coefficients / bc_ddim_coefficients; Euler is a = 1, b = dt, c = 0
@@ -327,7 +341,8 @@ bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t
  * rejected with INVALID_ARG before anything is enqueued.  cur, prev: device, n elements of
  * dtype, 16-byte aligned; out: 3 device doubles, as bc_probe_drift (same sums, within
  * rounding: the partial sums are grouped differently).  The first call on a device looks up
- * the array's device address (cudaGetSymbolAddress, with that device current); make that
+ * the array's device address (cudaGetSymbolAddress, with that device current), and so does
+ * the first call after the device's context was re-created (cudaDeviceReset); make that
  * first call before any stream capture.  Every call shares the one array; it keeps the last
  * call's partial sums, none of which a later call reads before rewriting them, so nothing
  * needs clearing, but calls that overlap on the device (on different streams, or from
@@ -342,7 +357,7 @@ bc_status bc_probe_drift_noalloc(const void *cur, const void *prev, int64_t n, b
 bc_status bc_cache_check(bc_handle h);
 
 /* Test hook for failure detection (no production use): what = 1 makes the next forecast
- * launch of this handle with H <= 3 run the pipeline kernel and leave the first stage of
+ * launch of this handle run the pipeline kernel and leave the first stage of
  * every CTA's pipeline unarmed, so that its bounded wait runs out (about one second) and the
  * launch returns early with the status word set, which bc_cache_check then reports;
  * what = 2 does the same to the next probe drift of at least one 16 KiB tile (its out[]

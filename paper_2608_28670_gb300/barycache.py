@@ -46,7 +46,8 @@ class bc_adaptive(ctypes.Structure):
 class bc_stats(ctypes.Structure):
     _fields_ = [("forecasts", ctypes.c_int64), ("pushes", ctypes.c_int64),
                 ("kernel_launches", ctypes.c_int64), ("memo_hits", ctypes.c_int64),
-                ("memo_misses", ctypes.c_int64), ("pipeline_launches", ctypes.c_int64)]
+                ("memo_misses", ctypes.c_int64), ("pipeline_launches", ctypes.c_int64),
+                ("table_uploads", ctypes.c_int64)]
 
 
 _lib = None

@@ -3,7 +3,8 @@
 Produces, next to this file under ``lib/``:
 
 * ``libbarycache.so`` -- the C-ABI forecast library (``include/barycache.h``): host solver,
-  cache manager and the grouped forecast / copy kernels.
+  cache manager and the grouped forecast / copy kernels (the forecast kernels compile as one
+  translation unit per history length, in parallel).
 * ``libbc_synth.so`` -- the seeded synthetic-input generator used by tests and benchmarks.
 
 Translation units compile in parallel; a unit is rebuilt only when a source or header is
@@ -29,11 +30,12 @@ COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fno-fast-math"
           "-I", INCLUDE, "-I", CSRC]
 
 LIBS = {
-    "libbarycache.so": ["bc_host.cpp", "bc_forecast.cu", "bc_probe.cu"],
+    "libbarycache.so": ["bc_host.cpp", "bc_forecast.cu", "bc_forecast_k1.cu", "bc_forecast_k2.cu",
+                        "bc_forecast_k3.cu", "bc_forecast_k4.cu", "bc_probe.cu"],
     "libbc_synth.so": ["bc_synth.cu"],
 }
 HEADERS = [os.path.join(INCLUDE, "barycache.h"), os.path.join(CSRC, "bc_internal.h"),
-           os.path.join(CSRC, "bc_tma.cuh")]
+           os.path.join(CSRC, "bc_tma.cuh"), os.path.join(CSRC, "bc_forecast_kernels.cuh")]
 
 
 def _newer(target: str, deps: list[str]) -> bool:

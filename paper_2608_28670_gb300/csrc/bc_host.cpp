@@ -214,6 +214,7 @@ struct bc_cache {
     Memo memo;
     bc_stats stats{};
     std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
+    bc::DeviceTable table;                        // device layer table (> 1016 layers only)
     double *probe_partials = nullptr;             // device scratch of bc_probe_drift
     uint32_t *status = nullptr;                   // device status word of the forecast kernels
     bool inject_next = false;                     // test hooks (bc_cache_inject_fault):
@@ -243,6 +244,48 @@ bc_status check_handle(bc_handle h) {
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The device layer table of a cache with more than kLayersLarge layers: n_layers entries of
+// device memory, the same of pinned host staging, and the event that orders reuse of the
+// staging after its last copy.
+bc_status alloc_table(bc_cache *h) {
+    bc::DeviceTable &tb = h->table;
+    const size_t bytes = sizeof(bc::LayerEntry) * static_cast<size_t>(h->n_layers);
+    void *dev = nullptr, *host = nullptr;
+    cudaEvent_t ev = nullptr;
+    cudaError_t e = cudaMalloc(&dev, bytes);
+    if (e == cudaSuccess) e = cudaHostAlloc(&host, bytes, cudaHostAllocDefault);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        if (dev) cudaFree(dev);
+        if (host) cudaFreeHost(host);
+        return e == cudaErrorMemoryAllocation ? fail(BC_ERR_OOM, "layer table")
+                                              : cuda_fail(e, "layer table");
+    }
+    tb.dev = static_cast<bc::LayerEntry *>(dev);
+    tb.host = static_cast<bc::LayerEntry *>(host);
+    tb.uploaded = ev;
+    tb.capacity = h->n_layers;
+    return BC_OK;
+}
+
+// Free every device and pinned allocation of the handle (the caller has synchronised).
+cudaError_t free_device(bc_cache *h) {
+    cudaError_t rc = cudaSuccess;
+    auto keep = [&rc](cudaError_t e) {
+        if (rc == cudaSuccess && e != cudaSuccess) rc = e;
+    };
+    if (h->arena) keep(cudaFree(h->arena));
+    if (h->probe_partials) keep(cudaFree(h->probe_partials));
+    if (h->table.dev) keep(cudaFree(h->table.dev));
+    if (h->table.host) keep(cudaFreeHost(h->table.host));
+    if (h->table.uploaded) keep(cudaEventDestroy(static_cast<cudaEvent_t>(h->table.uploaded)));
+    h->arena = nullptr;
+    h->probe_partials = nullptr;
+    h->table = bc::DeviceTable{};
+    return rc;
+}
 
 // Weights for a forecast at t_new from the live window (through the memo).
 bc_status window_weights(bc_cache *h, double t_new, double *c, int *m) {
@@ -282,6 +325,21 @@ struct Update {
 
 bool ranges_overlap(uint64_t a, uint64_t an, uint64_t b, uint64_t bn) {
     return an && bn && a < b + bn && b < a + an;
+}
+
+// The device layer table for a forecast of n_layers layers, or nullptr when the launch must
+// carry its tables in parameter blocks: few enough layers, no table on this handle, or a
+// stream that is being captured into a CUDA graph (a graph must hold every table it replays,
+// while the device table is rewritten by later calls).
+bc::DeviceTable *table_for(bc_cache *h, int n_layers, void *stream) {
+    if (n_layers <= bc::kLayersLarge || !h->table.dev || n_layers > h->table.capacity)
+        return nullptr;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(static_cast<cudaStream_t>(stream), &cs) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return cs == cudaStreamCaptureStatusNone ? &h->table : nullptr;
 }
 
 bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
@@ -344,10 +402,9 @@ bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dty
     }
 
     bc::LaunchPlan plan{};
-    for (int j = 0; j < BC_MAX_K; ++j) {
+    for (int j = 0; j < BC_MAX_K; ++j)
         plan.slot[j] = j < m ? reinterpret_cast<uint64_t>(h->slot_base(h->slot_of_node(j))) : 0;
-        plan.w[j] = j < m ? static_cast<float>(c[j]) : 0.0f;
-    }
+    bc::kernel_weights(c, m, plan.w, &plan.scale);
     plan.K = m;
     plan.in_dtype = h->dtype;
     plan.out_dtype = out_dtype;
@@ -367,6 +424,7 @@ bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dty
     if (plan.n_layers > 0) {
         DeviceGuard g(h->device);
         if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+        plan.table = table_for(h, plan.n_layers, stream);
         const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches,
                                                 &h->stats.pipeline_launches);
         h->inject_next = false;
@@ -507,6 +565,14 @@ bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype d
             h->probe_partials = static_cast<double *>(mem);
             h->status = reinterpret_cast<uint32_t *>(static_cast<char *>(mem) + scratch);
         }
+        if (n_layers > bc::kLayersLarge) {
+            s = alloc_table(h);
+            if (s != BC_OK) {
+                free_device(h);
+                delete h;
+                return s;
+            }
+        }
         {
             std::lock_guard<std::mutex> lk(g_registry_mu);
             g_registry.insert(h);
@@ -532,11 +598,10 @@ bc_status bc_cache_destroy(bc_handle h) {
     }
     h->magic = 0;
     bc_status rc = BC_OK;
-    if (h->arena || h->probe_partials) {
+    if (h->arena || h->probe_partials || h->table.dev) {
         DeviceGuard g(h->device);
         cudaError_t e = cudaDeviceSynchronize();
-        if (e == cudaSuccess && h->arena) e = cudaFree(h->arena);
-        if (e == cudaSuccess && h->probe_partials) e = cudaFree(h->probe_partials);
+        if (e == cudaSuccess) e = free_device(h);
         if (e != cudaSuccess) rc = cuda_fail(e, "cudaFree");
     }
     delete h;
@@ -808,11 +873,10 @@ bc_status bc_forecast_flat(bc_handle h, double t_new, void *out, void *stream) {
             e.dst = reinterpret_cast<uint64_t>(out);
             e.numel = static_cast<int64_t>(h->slot_bytes / elem_bytes(h->dtype));
             bc::LaunchPlan plan{};
-            for (int j = 0; j < BC_MAX_K; ++j) {
+            for (int j = 0; j < BC_MAX_K; ++j)
                 plan.slot[j] =
                     j < m ? reinterpret_cast<uint64_t>(h->slot_base(h->slot_of_node(j))) : 0;
-                plan.w[j] = j < m ? static_cast<float>(c[j]) : 0.0f;
-            }
+            bc::kernel_weights(c, m, plan.w, &plan.scale);
             plan.K = m;
             plan.in_dtype = h->dtype;
             plan.out_dtype = h->dtype;
@@ -956,6 +1020,7 @@ bc_status bc_cache_stats(bc_handle h, bc_stats *out) {
     if (!out) return fail(BC_ERR_INVALID_ARG, "out is NULL");
     h->stats.memo_hits = h->memo.hits;
     h->stats.memo_misses = h->memo.misses;
+    h->stats.table_uploads = h->table.uploads;
     *out = h->stats;
     return BC_OK;
 }

@@ -35,17 +35,20 @@ constexpr int kVecBytes = BC_VEC_BYTES;
 constexpr int kThreads = BC_THREADS;
 static_assert(kVecBytes == 16 || kVecBytes == 32, "vector loads are 16 or 32 bytes");
 
-// Independent vectors per thread and history slot for a K-term forecast.
+// Independent vectors per thread and history slot for a K-term forecast (register kernel).
 template <int K>
 constexpr int kVecsPerThreadFor = BC_VECS_PER_THREAD > 0 ? BC_VECS_PER_THREAD : (K >= 4 ? 4 : 2);
 // The push copy streams one source: four 16-byte vectors per thread.
 constexpr int kCopyVecsPerThread = 4;
 
 // Layers per launch carried in the kernel's parameter block.  The whole table travels as
-// a __grid_constant__ parameter, so a forecast needs no device-side scratch and no
-// host-to-device copy of its own; three table sizes keep the block small for the usual
-// few-dozen-layer caches, and caches with more than kLayersLarge layers issue one launch
-// per group.
+// a __grid_constant__ parameter, so a forecast of up to kLayersLarge layers needs no
+// device-side table and no host-to-device copy of its own; three table sizes keep the block
+// small for the usual few-dozen-layer caches.  A forecast over more layers runs as one
+// launch that reads its table from a per-handle device copy (DeviceTable); while its stream
+// is being captured into a CUDA graph it issues one parameter-block launch per kLayersLarge
+// layers instead, so that the graph holds every table it replays.  Push copies of more than
+// kLayersLarge layers always issue one launch per group.
 constexpr int kLayersSmall = 8;
 constexpr int kLayersMedium = 64;
 constexpr int kLayersLarge = 1016;
@@ -61,26 +64,44 @@ struct LayerEntry {        // 32 bytes
 template <int CAP>
 struct ForecastArgs {
     uint64_t slot[BC_MAX_K];  // slot base address of node j (j = 0 newest)
-    float w[BC_MAX_K];        // weights W_j rounded to fp32
+    float w[BC_MAX_K];        // weights W_j rounded to fp32, divided by `scale`
+    float scale;              // power of two >= sum_j |W_j|: the forecast is scale * sum_j w_j F_j
     float ca, cb, cc;         // sampler update x <- ca x + cb v_hat + cc z (update layer)
     int32_t n_layers;
-    int32_t euler_layer;      // index into `layer` of the update layer, or -1
+    int32_t euler_layer;      // index into the layer table of the update layer, or -1
     int32_t x_bf16;           // sampler state dtype (and z's): 1 = bf16, 0 = f32
     uint64_t x;               // sampler state address
     uint64_t z;               // noise address (0: no noise term)
     uint32_t *status;         // device status word: bit 0 = a pipeline wait timed out
     int32_t inject;           // test hook: leave the first pipeline stage unarmed
     int64_t total_tiles;
-    LayerEntry layer[CAP];
+    const LayerEntry *table;  // CAP == 0: the layer table in device memory
+    LayerEntry layer[CAP > 0 ? CAP : 1];  // CAP > 0: the layer table itself
 };
 
 // Kernel parameter blocks may hold up to 32,764 bytes (CUDA 12.1 and later).
 static_assert(sizeof(ForecastArgs<kLayersLarge>) <= 32764, "layer table exceeds the parameter block");
 
+// A device-memory copy of a launch's layer table, for forecasts over more layers than the
+// parameter block holds (one per handle; only caches of more than kLayersLarge layers have
+// one).  The table is uploaded from pinned staging with one cudaMemcpyAsync on the call's
+// stream, and only when it differs from the previous upload: a sampler that reuses its
+// output buffers uploads once.
+struct DeviceTable {
+    LayerEntry *dev = nullptr;     // device, `capacity` entries
+    LayerEntry *host = nullptr;    // pinned staging: the entries of the last upload
+    int capacity = 0;
+    int valid = 0;                 // entries of the last upload (0: none yet)
+    bool pending = false;          // `uploaded` was recorded after an upload
+    void *uploaded = nullptr;      // cudaEvent_t recorded after the last upload
+    int64_t uploads = 0;           // uploads so far
+};
+
 // Host-side view of one launch, independent of CAP.
 struct LaunchPlan {
     uint64_t slot[BC_MAX_K];
-    float w[BC_MAX_K];
+    float w[BC_MAX_K];        // fp32 weights divided by `scale` (see kernel_weights)
+    float scale;
     int K;                    // live nodes used (1..BC_MAX_K)
     bc_dtype in_dtype;
     bc_dtype out_dtype;
@@ -94,7 +115,29 @@ struct LaunchPlan {
     int kernel;               // bc_kernel choice: 0 auto, 1 register, 2 pipeline
     const LayerEntry *layers; // tile_end filled by the launcher
     int n_layers;
+    DeviceTable *table;       // non-null: more than kLayersLarge layers go in one launch
 };
+
+// Kernel weights from the fp64 weights c[0..m-1]: each is rounded to fp32 once, and all are
+// divided by the smallest power of two `scale` >= sum_j |fp32(c_j)| (at least 1).  The kernels
+// accumulate sum_j w_j F_j and multiply by `scale` at the end.  Scaling by a power of two is
+// exact, so wherever the unscaled fp32 sum neither overflows nor enters the subnormal range
+// the result is bit for bit the unscaled one; what it buys is that no partial sum exceeds
+// max_j |F_j| in magnitude, so finite inputs never overflow in fp32 where the exact
+// combination (weights near (3, -3, 1) or (4, -6, 4, -1) on values near the bf16 or fp32
+// maximum) is representable.
+inline void kernel_weights(const double *c, int m, float *w, float *scale) {
+    double sum = 0.0;
+    for (int j = 0; j < m; ++j) {
+        w[j] = static_cast<float>(c[j]);
+        sum += w[j] < 0.0f ? -static_cast<double>(w[j]) : static_cast<double>(w[j]);
+    }
+    float s = 1.0f;
+    while (static_cast<double>(s) < sum && s < 1073741824.0f) s *= 2.0f;
+    for (int j = 0; j < m; ++j) w[j] /= s;
+    for (int j = m; j < BC_MAX_K; ++j) w[j] = 0.0f;
+    *scale = s;
+}
 
 // Tiles needed for `numel` elements of `elem_bytes` each, in vectors of `vec_bytes`,
 // `tile_vecs` vectors per tile.
@@ -104,11 +147,21 @@ inline int64_t tiles_for(int64_t numel, int elem_bytes, int vec_bytes, int tile_
     return (vecs + tile_vecs - 1) / tile_vecs;
 }
 
-// Enqueue the grouped forecast (one launch per CAP-sized group of layers).  Returns the
-// CUDA error of the last launch; *launches is incremented per launch, *pipeline_launches
-// per launch of the shared-memory pipeline kernel.
+// Enqueue the grouped forecast: one launch, or with more than kLayersLarge layers and no
+// device table one launch per group of kLayersLarge.  Returns the CUDA error of the last
+// launch; *launches is incremented per launch, *pipeline_launches per launch of the
+// shared-memory pipeline kernel.
 int launch_forecast(const LaunchPlan &plan, void *stream, int64_t *launches,
                     int64_t *pipeline_launches);
+// The same for a given number of live nodes (bc_forecast_k{1,2,3,4}.cu).
+int launch_forecast_k1(const LaunchPlan &plan, void *stream, int64_t *launches,
+                       int64_t *pipeline_launches);
+int launch_forecast_k2(const LaunchPlan &plan, void *stream, int64_t *launches,
+                       int64_t *pipeline_launches);
+int launch_forecast_k3(const LaunchPlan &plan, void *stream, int64_t *launches,
+                       int64_t *pipeline_launches);
+int launch_forecast_k4(const LaunchPlan &plan, void *stream, int64_t *launches,
+                       int64_t *pipeline_launches);
 
 // Probe drift reduction (bc_probe.cu): at most kProbeMaxCtas partial pairs of scratch.
 constexpr int kProbeMaxCtas = 1024;

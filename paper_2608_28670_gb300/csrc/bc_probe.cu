@@ -18,6 +18,7 @@
 // element bf16 probe pair: 6.98 TB/s with five 2 x 16 KiB stages (four: 6.91, three: 6.75,
 // six: 6.80, 2 x 32 KiB stages x 2 / x 3: 6.91 / 6.73, eight 2 x 8 KiB: 5.16), register
 // loads 6.84.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -221,8 +222,10 @@ __global__ void __launch_bounds__(kProbeThreads)
                 const double nan = __longlong_as_double(0x7ff8000000000000LL);
                 partials[2 * blockIdx.x] = nan;
                 partials[2 * blockIdx.x + 1] = nan;
+                // the stage the test hook left unarmed (the first issued) has no copy
                 for (int64_t k = i; k < issued; ++k)
-                    mbar_wait_bounded(&full[k % S], static_cast<uint32_t>((k / S) & 1));
+                    if (!(inject && k == 0))
+                        mbar_wait_bounded(&full[k % S], static_cast<uint32_t>((k / S) & 1));
             }
             return;
         }
@@ -439,27 +442,73 @@ __global__ void __launch_bounds__(kProbeThreads)
 
 std::mutex g_static_mu;
 constexpr int kMaxDevices = 64;
-double *g_static_scratch[kMaxDevices] = {};
+
+// The looked-up address of g_drift_scratch per device, with the id of the context it was
+// looked up in: a context created later on the same device (after cudaDeviceReset, say)
+// loads the library's module afresh, at a possibly different address.
+struct StaticScratch {
+    double *ptr = nullptr;
+    unsigned long long ctx = 0;
+};
+StaticScratch g_static_scratch[kMaxDevices];
+
+// Unique id of the calling thread's current context (the driver's cuCtxGetId, reached through
+// the runtime's entry-point query so that the library does not link the driver API), or 0
+// when no context is current or the query is unavailable.  Called with g_static_mu held.
+unsigned long long current_context_id() {
+    using GetCurrent = CUresult (*)(CUcontext *);
+    using GetId = CUresult (*)(CUcontext, unsigned long long *);
+    static bool tried = false;
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    if (!tried) {
+        tried = true;
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(f);
+        f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(f);
+        cudaGetLastError();
+    }
+    if (!get_current || !get_id) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+    if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
 
 // Device address of g_drift_scratch on the current device.  In host code the array's name
-// only stands in for the symbol, so the address is looked up with cudaGetSymbolAddress,
-// once per device, with that device current (the first no-allocation call on it).
+// only stands in for the symbol, so the address is looked up with cudaGetSymbolAddress, with
+// that device current: on the first no-allocation call on a device, and again whenever the
+// device's current context is not the one the address was looked up in (or cannot be told).
 int static_scratch(double **out) {
     int dev = 0;
     int err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lk(g_static_mu);
-    if (!g_static_scratch[dev]) {
-        void *p = nullptr;
-        err = cudaGetSymbolAddress(&p, g_drift_scratch);
-        if (err != cudaSuccess) {
-            cudaGetLastError();  // reported once, by return value
-            return err;
-        }
-        g_static_scratch[dev] = static_cast<double *>(p);
+    StaticScratch &sc = g_static_scratch[dev];
+    const unsigned long long ctx = current_context_id();
+    if (sc.ptr && ctx != 0 && sc.ctx == ctx) {
+        *out = sc.ptr;
+        return cudaSuccess;
     }
-    *out = g_static_scratch[dev];
+    void *p = nullptr;
+    err = cudaGetSymbolAddress(&p, g_drift_scratch);
+    if (err != cudaSuccess) {
+        cudaGetLastError();  // reported once, by return value
+        return err;
+    }
+    sc.ptr = static_cast<double *>(p);
+    sc.ctx = current_context_id();  // the lookup made the device's context current
+    *out = sc.ptr;
     return cudaSuccess;
 }
 

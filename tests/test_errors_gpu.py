@@ -118,21 +118,23 @@ def test_degenerate_weights_status():
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("K", [3, 4])
 @pytest.mark.parametrize("flat", [False, True])
-def test_pipeline_wait_timeout_is_reported_and_recovers(flat):
+def test_pipeline_wait_timeout_is_reported_and_recovers(flat, K):
     """Failure detection on the device: the test hook leaves each CTA's first pipeline stage
     unarmed, so the forecast kernel's bounded wait runs out (about a second); the launch
     returns, bc_cache_check reports BC_ERR_DEVICE_TIMEOUT once, and the next forecast on the
-    same handle and context is correct."""
+    same handle and context is correct.  The drain after the timeout skips the unarmed stage,
+    so the whole launch gives up after one wait limit, not two."""
     import time
     import numpy as np
     import oracle
     from paper_2608_28670_gb300 import synth
     from tests.gpu_helpers import assert_close, to_device, to_host
     numels = [100_000, 3 * 8192 + 5]
-    times = [0.9, 0.85, 0.8]
+    times = [0.9, 0.85, 0.8, 0.775][:K]
     feats = synth.host_trajectories([(n,) for n in numels], times, dtype="bf16", seed=44)
-    h = bc.bc_cache_create(numels, 3, bc.DTYPE_BF16)
+    h = bc.bc_cache_create(numels, K, bc.DTYPE_BF16)
     try:
         for t, per in zip(times, feats):
             dev = [to_device(f) for f in per]
@@ -153,12 +155,12 @@ def test_pipeline_wait_timeout_is_reported_and_recovers(flat):
         t0 = time.perf_counter()
         forecast()
         assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
-        assert 0.5 < time.perf_counter() - t0 < 60.0
+        assert 0.5 < time.perf_counter() - t0 < 1.9
         bc.bc_cache_check(h)                         # reported once, then clear
         forecast()                                   # the handle and context still work
         bc.bc_cache_check(h)
         torch.cuda.synchronize()
-        W = oracle.paper_weights([0.8, 0.85, 0.9], 0.75)
+        W = oracle.paper_weights(times[::-1], 0.75)
         nf = feats[::-1]
         host_flat = to_host(flat_out, bc.DTYPE_BF16)
         for l, n in enumerate(numels):
@@ -190,7 +192,7 @@ def test_drift_pipeline_wait_timeout_is_reported_and_recovers():
         t0 = time.perf_counter()
         bc.bc_probe_drift(h, c.data_ptr(), p.data_ptr(), n, bc.DTYPE_F32, out.data_ptr(), s())
         assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
-        assert 0.5 < time.perf_counter() - t0 < 60.0
+        assert 0.5 < time.perf_counter() - t0 < 1.9
         assert np.isnan(out.cpu().numpy()).all()
         bc.bc_cache_check(h)
         bc.bc_probe_drift(h, c.data_ptr(), p.data_ptr(), n, bc.DTYPE_F32, out.data_ptr(), s())
@@ -214,7 +216,7 @@ def test_push_pipeline_wait_timeout_is_reported_and_recovers():
         t0 = time.perf_counter()
         bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())
         assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
-        assert 0.5 < time.perf_counter() - t0 < 60.0
+        assert 0.5 < time.perf_counter() - t0 < 1.9
         bc.bc_cache_check(h)
         bc.bc_cache_reset(h)
         bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())

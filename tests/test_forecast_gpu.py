@@ -21,7 +21,8 @@ from tests.gpu_helpers import (as_f64, assert_close, device_view, empty_out, ora
 pytestmark = pytest.mark.gpu
 
 DT_NAME = {bc.DTYPE_F32: "f32", bc.DTYPE_BF16: "bf16"}
-# A tile holds 16 KiB of each history slot (32 KiB at K = 4): 8192 bf16 / 4096 f32 elements.
+# A tile holds 16 KiB of each history slot (32 KiB at K = 4 in the register kernel, 8 KiB in
+# small launches): 8192 bf16 / 4096 f32 elements.
 RAGGED = [1, 7, 8, 9, 4095, 4096, 4097, 8191, 8192, 8193, 3 * 8192 + 5, 100_003]
 
 
@@ -132,7 +133,7 @@ def test_zero_copy_push(kernel):
     bc.bc_cache_destroy(h)
 
 
-@pytest.mark.parametrize("K", [1, 2, 3])
+@pytest.mark.parametrize("K", [1, 2, 3, 4])
 @pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 @pytest.mark.parametrize("out_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 def test_register_and_pipeline_kernels_agree_bitwise(K, in_dt, out_dt):
@@ -240,16 +241,102 @@ def test_null_outputs_skip_layers_and_window_forecast():
         bc.bc_cache_destroy(h)
 
 
-def test_many_layers_use_several_launches():
-    numels = [(i * 37) % 301 + 1 for i in range(1100)]   # 1100 tiny ragged layers
+def test_many_layers_one_launch_through_the_device_table():
+    # 1100 tiny ragged layers: more than one parameter block holds, so the layer table goes to
+    # the handle's device copy and the forecast is one launch (run_case checks every layer
+    # against the oracle).  The table is uploaded once for a set of outputs and again only
+    # when the outputs change.
+    numels = [(i * 37) % 301 + 1 for i in range(1100)]
     times = [0.9, 0.85]
     h = run_case(numels, 2, 2, bc.DTYPE_F32, bc.DTYPE_BF16, bc.make_params(), 0.8, times, seed=9)
     try:
-        s0 = bc.bc_cache_stats(h)["kernel_launches"]
+        st0 = bc.bc_cache_stats(h)
+        assert st0["table_uploads"] == 1
         outs = [empty_out(n, bc.DTYPE_BF16) for n in numels]
-        bc.bc_forecast(h, 0.8, [o.data_ptr() for o in outs], bc.DTYPE_BF16, stream())
+        ptrs = [o.data_ptr() for o in outs]
+        for _ in range(3):
+            bc.bc_forecast(h, 0.8, ptrs, bc.DTYPE_BF16, stream())
         torch.cuda.synchronize()
-        assert bc.bc_cache_stats(h)["kernel_launches"] - s0 == 2   # 1016 + 84 layers
+        st1 = bc.bc_cache_stats(h)
+        assert st1["kernel_launches"] - st0["kernel_launches"] == 3     # one per call
+        assert st1["table_uploads"] == 2                                 # new outputs: once
+        first = [o.clone() for o in outs]
+        ptrs2 = list(ptrs)
+        ptrs2[5] = None                                                  # a different table
+        outs[7].fill_(0)
+        bc.bc_forecast(h, 0.8, ptrs2, bc.DTYPE_BF16, stream())
+        bc.bc_forecast(h, 0.8, ptrs, bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["table_uploads"] == 4
+        for a, b in zip(first, outs):
+            assert torch.equal(a, b)
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+def test_many_layers_in_a_graph_carry_their_own_tables(kernel):
+    # While the stream is captured, a forecast over more layers than one parameter block holds
+    # is split into parameter-block launches, so the graph does not depend on the device table
+    # that later calls rewrite.  Replaying it after an eager call with other outputs must
+    # still write the captured outputs, bit for bit as the eager one-launch forecast.
+    numels = [(i * 53) % 977 + 8 for i in range(2100)]
+    times = [0.9, 0.85, 0.8]
+    h = run_case(numels, 3, 3, bc.DTYPE_BF16, bc.DTYPE_BF16, bc.make_params(), 0.75, times,
+                 seed=12, kernel=kernel)
+    try:
+        outs = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        eager = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        # first uses of the parameter-block launchers (1016- and 64-entry tables) outside the
+        # capture, as the header asks
+        for sel in (1000, 60):
+            bc.bc_forecast(h, 0.75, [o.data_ptr() if l < sel else None
+                                     for l, o in enumerate(eager)], bc.DTYPE_BF16, stream())
+        bc.bc_forecast(h, 0.75, [o.data_ptr() for o in eager], bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        with torch.cuda.stream(s):
+            l0 = bc.bc_cache_stats(h)["kernel_launches"]
+            with torch.cuda.graph(g, stream=s, capture_error_mode="thread_local"):
+                bc.bc_forecast(h, 0.75, [o.data_ptr() for o in outs], bc.DTYPE_BF16,
+                               s.cuda_stream)
+            assert bc.bc_cache_stats(h)["kernel_launches"] - l0 == 3    # 1016 + 1016 + 68
+        other = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        bc.bc_forecast(h, 0.75, [o.data_ptr() for o in other], bc.DTYPE_BF16, stream())
+        for o in outs:
+            o.fill_(0)
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        for a, b in zip(eager, outs):
+            assert torch.equal(a, b)
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+@pytest.mark.parametrize("K", [1, 2, 3, 4])
+def test_small_launch_half_tiles_match_the_register_kernel(in_dt, K):
+    # A launch of fewer than two tiles per SM runs the register kernel with half-size tiles
+    # under AUTO; pinning REGISTER keeps the full tiles.  Same per-element arithmetic: the
+    # outputs must agree bit for bit (and run_case has checked AUTO against the oracle).
+    numels = [2 * 256 * 1152, 4097, 13]
+    times = [0.9 - 0.05 * i for i in range(K)]
+    h = run_case(numels, K, K, in_dt, in_dt, bc.make_params(), times[-1] - 0.05, times,
+                 seed=31 + K)
+    try:
+        res = []
+        for kern in (bc.KERNEL_AUTO, bc.KERNEL_REGISTER):
+            bc.bc_cache_set_kernel(h, kern)
+            outs = [empty_out(n, in_dt) for n in numels]
+            bc.bc_forecast(h, times[-1] - 0.05, [o.data_ptr() for o in outs], in_dt, stream())
+            torch.cuda.synchronize()
+            res.append(outs)
+        for a, b in zip(*res):
+            assert torch.equal(a, b)
     finally:
         bc.bc_cache_destroy(h)
 
