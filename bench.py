@@ -63,6 +63,9 @@ def parse_args():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-extra", action="store_true",
                     help="skip the push and fused-step measurements")
+    ap.add_argument("--kernel", choices=["auto", "register", "pipeline"], default="auto",
+                    help="pin the forecast kernel of the headline leg (default: the library's "
+                         "choice)")
     return ap.parse_args()
 
 
@@ -77,6 +80,11 @@ def measured_peak():
 
 
 KERNEL_CODE_END = "// ------------------------------------------------------------------ launch plumbing"
+# Warm-up lasts at least this long (wall time) as well as the requested number of steps:
+# freeing a very large allocation (a previous leg's cache) costs HBM bandwidth for a while
+# afterwards (about 70 ms after freeing 170 GB, at ~5.0 instead of ~7.1 TB/s), and a leg
+# of short launches would otherwise time that transient.
+MIN_WARMUP_S = 0.25
 
 
 def _code_only(src: bytes) -> bytes:
@@ -90,12 +98,13 @@ def _code_only(src: bytes) -> bytes:
 
 
 def kernel_source_hash() -> str:
-    """Hash of the forecast kernels' device code (bc_forecast.cu up to its host launch
-    plumbing) and of the headers it includes from the package (layout, pipeline primitives),
-    comments and whitespace ignored: a change there voids a stored ncu figure."""
+    """Hash of the forecast kernels' device code (bc_forecast_kernels.cuh up to its host
+    launch plumbing, the tuning macros included) and of the headers it includes from the
+    package (layout, pipeline primitives), comments and whitespace ignored: a change there
+    voids a stored ncu figure."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_28670_gb300", "csrc")
-    with open(os.path.join(csrc, "bc_forecast.cu"), "rb") as fh:
+    with open(os.path.join(csrc, "bc_forecast_kernels.cuh"), "rb") as fh:
         h.update(_code_only(fh.read().split(KERNEL_CODE_END.encode(), 1)[0]))
     for name in ("bc_internal.h", "bc_tma.cuh"):
         with open(os.path.join(csrc, name), "rb") as fh:
@@ -103,9 +112,12 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str, K: int):
-    """DRAM bytes per output element of the forecast kernel from the committed ncu summary, if
-    it was taken on this workload, K and the current kernel source (else None)."""
+def profiled_traffic(K: int, kernel: str, io: str = "bf16/bf16"):
+    """DRAM bytes per output element of the forecast kernel (`kernel`: "pipeline" or
+    "register") at history length K, from the committed ncu record, if one was taken with
+    the current kernel source (else None).  The record comes from a small case (a few GB of
+    cache); a launch moves the same bytes per element whatever its size, so the bench scales
+    it by the elements of its own launch."""
     path = os.path.join(ROOT, "profiles", "forecast_kernel_traffic.json.txt")
     try:
         with open(path) as fh:
@@ -114,10 +126,8 @@ def profiled_traffic(workload: str, K: int):
         return None
     if rec.get("kernel_source_sha256_16") != kernel_source_hash():
         return None
-    if rec.get("workload") != workload:
-        return None
-    per_elem = rec.get("dram_bytes_per_output_element", {}).get(f"K{K}")
-    return per_elem
+    entry = rec.get("records", {}).get(f"K{K}/{kernel}/{io}")
+    return entry.get("dram_bytes_per_output_element") if entry else None
 
 
 class ClockSampler:
@@ -231,6 +241,24 @@ def window_targets(w, K):
     return ts or [rep.t]
 
 
+def warm_up(step, count, min_s=MIN_WARMUP_S):
+    """Run `step(i)` at least `count` times and for at least `min_s` seconds of wall time
+    (synchronised); returns the number of steps run."""
+    import torch
+    t0 = time.perf_counter()
+    i = 0
+    while i < count:
+        step(i)
+        i += 1
+    torch.cuda.synchronize()
+    while time.perf_counter() - t0 < min_s:
+        for _ in range(4):
+            step(i)
+            i += 1
+        torch.cuda.synchronize()
+    return i
+
+
 def time_forecast(run, steps, warmup, stream, dist=None):
     """Time `steps` skipped steps.  A workload whose step moves less than four L2s of data
     would be served from L2 back to back, so then L2 is flushed (a 512 MB write) before every
@@ -241,9 +269,7 @@ def time_forecast(run, steps, warmup, stream, dist=None):
     if run.algorithmic_bytes() < 4 * L2_BYTES:
         flush = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda")
     with nvtx_range("warmup"):
-        for i in range(warmup):
-            run.forecast(ts[i % len(ts)])
-        torch.cuda.synchronize()
+        warm_up(lambda i: run.forecast(ts[i % len(ts)]), warmup)
     if dist is not None:
         dist.barrier()
     st0 = run.stats()
@@ -302,6 +328,9 @@ def run_ours(args):
     stream = torch.cuda.current_stream().cuda_stream
 
     run = WorkloadRun(w, K=K, budget_bytes=budget, stream=stream)
+    kernel_choice = {"auto": bc.KERNEL_AUTO, "register": bc.KERNEL_REGISTER,
+                     "pipeline": bc.KERNEL_PIPELINE}[args.kernel]
+    bc.bc_cache_set_kernel(run.h, kernel_choice)
     try:
         torch.cuda.synchronize()
         clocks = ClockSampler(not args.no_clocks)
@@ -316,7 +345,9 @@ def run_ours(args):
         per_launch_bytes = alg / max(launches_per_step, 1)
         peak, peak_kind = measured_peak()
         achieved = per_launch_bytes / (kernel_ms * 1e-3) / 1e9
-        traffic_per_elem = profiled_traffic(w.name, K)
+        kernel_kind = "pipeline" if time_forecast.pipeline == launches else "register"
+        io = "bf16/bf16" if w.dtype == bc.DTYPE_BF16 else "f32/f32"
+        traffic_per_elem = None if w.euler_shape else profiled_traffic(K, kernel_kind, io)
         per_launch_elems = elems / max(launches_per_step, 1)
         result = {
             "metric": METRIC, "value": round(value, 1), "unit": "GB/s",
@@ -333,6 +364,8 @@ def run_ours(args):
                 "weights": "paper Eqs. 8-12, delta_H table, lambda 0, C 10, eta 1e-12",
                 "targets": window_targets(w, K), "nodes": list(run.problem.nodes),
                 "l2": time_forecast.l2,
+                "kernel_choice": args.kernel,
+                "warmup_s_min": MIN_WARMUP_S,
                 "parallelism": f"replicas x{world}",
             },
             "pct_of_measured_peak": round(100 * value / world / peak, 2),
@@ -344,10 +377,17 @@ def run_ours(args):
             "roofline": {
                 "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                 "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+                "nominal_peak": NOMINAL_HBM_GBS,
+                "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
                 "traffic": (round(traffic_per_elem * per_launch_elems)
                             if traffic_per_elem else None),
+                "traffic_source": ("ncu dram__bytes_read.sum + dram__bytes_write.sum per output "
+                                   "element on t2i-1024-shaped launches (profiles/"
+                                   "forecast_kernel_traffic.json.txt), times this launch's "
+                                   "output elements" if traffic_per_elem else
+                                   "no ncu record for this kernel source, K and kernel"),
                 "kernel": ("bc::forecast_tma_kernel (TMA pipeline)"
-                           if time_forecast.pipeline == launches else "bc::forecast_kernel"),
+                           if kernel_kind == "pipeline" else "bc::forecast_kernel"),
                 "avg_launch_ms": round(kernel_ms, 4),
                 "algorithmic_bytes_per_launch": per_launch_bytes,
             },
@@ -366,14 +406,24 @@ def run_ours(args):
             torch.cuda.empty_cache()
             for k in w.K_sweep:
                 r = WorkloadRun(w, K=k, budget_bytes=budget, stream=stream)
+                bc.bc_cache_set_kernel(r.h, kernel_choice)
                 try:
                     tm, ps, ln = time_forecast(r, args.steps, args.warmup, stream, dist)
                     a = r.algorithmic_bytes()
                     m = tm / args.steps
-                    sweep[f"K{k}"] = {"GB/s": round(a / (m * 1e-3) / 1e9, 1), "ms": round(m, 4),
+                    kk = "pipeline" if time_forecast.pipeline == ln else "register"
+                    per = profiled_traffic(k, kk, io)
+                    lpl = ln / args.steps                       # launches per step
+                    gbs = a / (m * 1e-3) / 1e9
+                    sweep[f"K{k}"] = {"GB/s": round(gbs, 1), "ms": round(m, 4),
+                                      "frac": round(gbs / peak, 4),
+                                      "frac_of_nominal": round(gbs / NOMINAL_HBM_GBS, 4),
                                       "cache_bytes": bc.bc_cache_bytes(r.h),
                                       "calls_per_step": r.calls, "layers_per_call": r.window,
-                                      "launches": ln}
+                                      "launches": ln, "kernel": kk,
+                                      "algorithmic_bytes_per_launch": a / lpl,
+                                      "traffic": (round(per * r.w.layer_numel * r.n_feat / lpl)
+                                                  if per else None)}
                 finally:
                     r.close()
                     torch.cuda.empty_cache()
@@ -395,10 +445,11 @@ def run_ours(args):
     finally:
         if run is not None:
             run.close()
+    cpu_legs = rank == 0 and world == 1 and not args.no_cpu_baseline
     if not args.no_extra and w.name != "mmdit-t2i":
         torch.cuda.empty_cache()
         with nvtx_range("fused_step"):
-            result["fused_step"] = time_fused(args, stream, dist)
+            result["fused_step"] = time_fused(args, stream, dist, cpu=cpu_legs)
     if not args.no_extra:
         torch.cuda.empty_cache()
         with nvtx_range("sampling_loop"):
@@ -410,7 +461,7 @@ def run_ours(args):
             result["blockwise"] = time_blockwise(stream, args.steps)
         torch.cuda.empty_cache()
         with nvtx_range("other_workloads"):
-            result["other_workloads"] = time_other_workloads(stream, args.steps)
+            result["other_workloads"] = time_other_workloads(stream, args.steps, cpu=cpu_legs)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -439,26 +490,29 @@ def time_push(run, steps):
         return None
     ptrs = [o.data_ptr() for o in run.outs]
     slot = sum(n * run.w.elem_bytes for n in run.numels)
-    t = [_continuation(run, 100 + i)[0] for i in range(3 * (steps + 2))]
+    counter = [100]
 
-    def timed(kernel, k0):
+    def push(_i=0):
+        bc.bc_cache_push(run.h, ptrs, _continuation(run, counter[0])[0], run.stream)
+        counter[0] += 1
+
+    def timed(kernel):
         bc.bc_cache_set_kernel(run.h, kernel)
-        for i in range(2):
-            bc.bc_cache_push(run.h, ptrs, t[k0 + i], run.stream)
+        warm_up(push, 2)
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
         a.record()
         for i in range(steps):
-            bc.bc_cache_push(run.h, ptrs, t[k0 + 2 + i], run.stream)
+            push()
         b.record()
         torch.cuda.synchronize()
         return a.elapsed_time(b) / steps
 
     gbs = lambda ms: round(2 * slot / (ms * 1e-3) / 1e9, 1)
-    by_kernel = {"register": gbs(timed(bc.KERNEL_REGISTER, 0)),
-                 "pipeline": gbs(timed(bc.KERNEL_PIPELINE, steps + 2))}
-    ms = timed(bc.KERNEL_AUTO, 2 * (steps + 2))
+    by_kernel = {"register": gbs(timed(bc.KERNEL_REGISTER)),
+                 "pipeline": gbs(timed(bc.KERNEL_PIPELINE))}
+    ms = timed(bc.KERNEL_AUTO)
     bc.bc_cache_check(run.h)
     return {"GB/s": gbs(ms), "ms": round(ms, 4), "GB/s_by_kernel": by_kernel,
             "bytes_per_push": 2 * slot, "pushes": steps,
@@ -480,8 +534,8 @@ def time_probe(run, steps, probe_elems=None):
     cur = bc.bc_cache_slot_ptrs(run.h, 0, len(run.numels))[0]
     prev = bc.bc_cache_slot_ptrs(run.h, 1, len(run.numels))[0]
     out = torch.empty(3, dtype=torch.float64, device="cuda")
-    for _ in range(3):
-        bc.bc_probe_drift(run.h, cur, prev, n, run.w.dtype, out.data_ptr(), run.stream)
+    warm_up(lambda i: bc.bc_probe_drift(run.h, cur, prev, n, run.w.dtype, out.data_ptr(),
+                                        run.stream), 3)
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
@@ -647,8 +701,9 @@ def time_graph_loop(stream):
 
 def time_blockwise(stream, steps):
     """Row f2: a many-tensor (blockwise) cache -- 4096 tensors of 65,536 bf16 elements, K = 3
-    (1.6 GB of cache) -- forecast through per-layer output pointers (1016 layers per launch)
-    and through one flat slot-shaped output (one launch)."""
+    (1.6 GB of cache) -- forecast through per-layer output pointers (one launch reading its
+    layer table from the handle's device copy, uploaded once for these outputs) and through
+    one flat slot-shaped output (one launch)."""
     import numpy as np
     import torch
     from paper_2608_28670_gb300 import barycache as bc
@@ -669,16 +724,17 @@ def time_blockwise(stream, steps):
         alg = (3 * 2 + 2) * n * n_t
 
         def timed(fn):
-            for _ in range(3):
-                fn()
+            warm_up(lambda i: fn(), 3)
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
             torch.cuda.synchronize()
+            l0 = bc.bc_cache_stats(h)["kernel_launches"]
             a.record()
             for _ in range(steps):
                 fn()
             b.record()
             torch.cuda.synchronize()
+            timed.launches = (bc.bc_cache_stats(h)["kernel_launches"] - l0) / steps
             return a.elapsed_time(b) / steps
         by_kernel = {}
         for name, kern in (("register", bc.KERNEL_REGISTER), ("pipeline", bc.KERNEL_PIPELINE),
@@ -686,29 +742,30 @@ def time_blockwise(stream, steps):
             bc.bc_cache_set_kernel(h, kern)
             by_kernel[name] = round(alg / (timed(
                 lambda: bc.bc_forecast(h, 0.75, per, bc.DTYPE_BF16, stream)) * 1e-3) / 1e9, 1)
-        l0 = bc.bc_cache_stats(h)["kernel_launches"]
         ms_layers = timed(lambda: bc.bc_forecast(h, 0.75, per, bc.DTYPE_BF16, stream))
-        l1 = bc.bc_cache_stats(h)["kernel_launches"]
+        per_layer_launches = timed.launches
+        st = bc.bc_cache_stats(h)
         ms_flat = timed(lambda: bc.bc_forecast_flat(h, 0.75, flat.data_ptr(), stream))
-        l2 = bc.bc_cache_stats(h)["kernel_launches"]
         return {"tensors": n_t, "elements_per_tensor": n,
                 "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
                               "ms": round(ms_layers, 4),
-                              "launches_per_call": (l1 - l0) // (steps + 3),
+                              "launches_per_call": per_layer_launches,
+                              "table_uploads": st["table_uploads"],
                               "GB/s_by_kernel": by_kernel},
                 "flat": {"GB/s": round(alg / (ms_flat * 1e-3) / 1e9, 1), "ms": round(ms_flat, 4),
-                         "launches_per_call": (l2 - l1) // (steps + 3)}}
+                         "launches_per_call": timed.launches}}
     finally:
         bc.bc_cache_destroy(h)
 
 
-def time_other_workloads(stream, steps):
+def time_other_workloads(stream, steps, cpu=False):
     """The remaining workloads: c2i-256 (9.4 MB per forecast, L2-resident, so L2 is flushed
     by writing 512 MB before every timed launch, outside its event pair; the flush keeps the
     device busy while the host enqueues the forecast), c2i-512 (K = 4, 2.6 GB) and t2i-1024
     (K = 3, 4.2 GB), whose inputs exceed L2: `steps` forecasts back to back between one event
     pair, as in the headline measurement.  `idle_start_us` is one call on an idle device
-    (host call to completion: memo lookup, table build and launch latency included)."""
+    (host call to completion: memo lookup, table build and launch latency included).  With
+    `cpu`, each entry also carries the oracle over the whole workload (cpu_baseline_full)."""
     import torch
     from paper_2608_28670_gb300.configs import WORKLOADS
     from paper_2608_28670_gb300.runner import WorkloadRun
@@ -722,9 +779,8 @@ def time_other_workloads(stream, steps):
         w = WORKLOADS[name]
         r = WorkloadRun(w, stream=stream)
         try:
-            for _ in range(3):
-                r.forecast()
-            torch.cuda.synchronize()
+            warm_up(lambda i: r.forecast(), 3)
+            p0 = r.stats()["pipeline_launches"]
             if name == "c2i-256":
                 ms = []
                 for i in range(steps):
@@ -744,6 +800,7 @@ def time_other_workloads(stream, steps):
                 b.record()
                 torch.cuda.synchronize()
                 m = a.elapsed_time(b) / steps
+            pipe = r.stats()["pipeline_launches"] - p0
             idle = []
             for _ in range(5):
                 torch.cuda.synchronize()
@@ -753,21 +810,31 @@ def time_other_workloads(stream, steps):
                 b.record()
                 torch.cuda.synchronize()
                 idle.append(a.elapsed_time(b))
-            st = r.stats()
-            out[name] = {"GB/s": round(r.algorithmic_bytes() / (m * 1e-3) / 1e9, 1),
-                         "us": round(1e3 * m, 1), "bytes": r.algorithmic_bytes(),
+            gbs = r.algorithmic_bytes() / (m * 1e-3) / 1e9
+            out[name] = {"GB/s": round(gbs, 1), "us": round(1e3 * m, 1),
+                         "bytes": r.algorithmic_bytes(),
+                         "elems_per_s": round(r.w.layer_numel * r.n_feat / (m * 1e-3), 1),
                          "idle_start_us": round(1e3 * statistics.median(idle), 1),
-                         "K": r.K, "pipeline_kernel": st["pipeline_launches"] > 0,
+                         "K": r.K, "pipeline_kernel": pipe > 0,
+                         "cache_bytes": bc_cache_bytes(r),
                          "l2": "flushed before each launch" if name == "c2i-256"
                                else "inputs larger than L2, launches back to back"}
+            if cpu:
+                out[name]["cpu_baseline"] = cpu_baseline_full(r)
         finally:
             r.close()
     return out
 
 
-def time_fused(args, stream, dist):
+def bc_cache_bytes(run):
+    from paper_2608_28670_gb300 import barycache as bc
+    return bc.bc_cache_bytes(run.h)
+
+
+def time_fused(args, stream, dist, cpu=False):
     """Row a4: the fused forecast + Euler step on the MMDiT workload (57 block outputs plus
-    the velocity [1, 16, 128, 128], one launch per step)."""
+    the velocity [1, 16, 128, 128], one launch per step); with `cpu`, the oracle over the
+    whole step beside it."""
     from paper_2608_28670_gb300.configs import WORKLOADS
     from paper_2608_28670_gb300.runner import WorkloadRun
     r = WorkloadRun(WORKLOADS["mmdit-t2i"], stream=stream)
@@ -775,9 +842,13 @@ def time_fused(args, stream, dist):
         tm, ps, ln = time_forecast(r, args.steps, args.warmup, stream, dist)
         ms = tm / args.steps
         a = r.algorithmic_bytes()
-        return {"workload": "mmdit-t2i", "GB/s": round(a / (ms * 1e-3) / 1e9, 1),
-                "ms": round(ms, 4), "algorithmic_bytes_per_step": a, "launches": ln,
-                "steps": args.steps}
+        res = {"workload": "mmdit-t2i", "GB/s": round(a / (ms * 1e-3) / 1e9, 1),
+               "ms": round(ms, 4), "algorithmic_bytes_per_step": a, "launches": ln,
+               "elems_per_s": round(sum(r.numels) / (ms * 1e-3), 1),
+               "cache_bytes": bc_cache_bytes(r), "steps": args.steps}
+        if cpu:
+            res["cpu_baseline"] = cpu_baseline_full(r)
+        return res
     finally:
         r.close()
 
@@ -991,28 +1062,39 @@ def _oracle_task(args):
 
 class OraclePool:
     """The unmodified fp64 oracle on every host core: a spawn pool of one worker per core,
-    each running oracle.combine on chunks of a sample held in shared memory."""
+    each running oracle.combine on chunks of a sample held in shared memory.  `capacity`
+    (elements per node) sizes the shared block for later samples given to load()."""
 
-    def __init__(self, sample: list, W, workers: int | None = None):
+    def __init__(self, sample: list, W, workers: int | None = None,
+                 capacity: int | None = None):
         import multiprocessing as mp
         from multiprocessing import shared_memory
-        import numpy as np
         self.m = len(sample)
         self.dtype = sample[0].dtype
-        self.total = sample[0].size
-        self.shm = shared_memory.SharedMemory(create=True,
-                                              size=self.m * self.total * sample[0].itemsize)
-        arr = np.ndarray((self.m, self.total), dtype=self.dtype, buffer=self.shm.buf)
-        for j in range(self.m):
-            arr[j] = sample[j]
-        del arr
+        self.capacity = max(capacity or 0, sample[0].size)
+        self.shm = shared_memory.SharedMemory(
+            create=True, size=max(1, self.m * self.capacity * sample[0].itemsize))
         self.W = [float(w) for w in W]
         self.workers = workers or os.cpu_count() or 1
         self.pool = mp.get_context("spawn").Pool(self.workers, initializer=_oracle_pool_init)
-        self.tasks = [(self.shm.name, self.dtype, self.m, self.total, off,
-                       min(CHUNK, self.total - off), self.W)
-                      for off in range(0, self.total, CHUNK)]
+        self.load(sample)
         self.pool.map(_oracle_task, self.tasks[:self.workers])        # warm the workers
+
+    def load(self, sample: list):
+        """Copy a new sample (same node count and dtype, at most `capacity` elements per
+        node) into the shared block."""
+        import numpy as np
+        assert len(sample) == self.m and sample[0].dtype == self.dtype
+        total = sample[0].size
+        assert total <= self.capacity
+        arr = np.ndarray((self.m, self.capacity), dtype=self.dtype, buffer=self.shm.buf)
+        for j in range(self.m):
+            arr[j, :total] = sample[j]
+        del arr
+        self.total = total
+        self.tasks = [(self.shm.name, self.dtype, self.m, self.capacity, off,
+                       min(CHUNK, total - off), self.W)
+                      for off in range(0, total, CHUNK)]
 
     def run(self, passes: int = 1):
         """Process the whole sample `passes` times; returns (elements, seconds)."""
@@ -1091,6 +1173,97 @@ def cpu_baseline_from_device(run, seconds):
                       f"times by {cores} spawned workers running the fp64 oracle, {secs:.1f} s",
             "single_core": {"value": round(n1 * per_elem / t1 / 1e9, 4), "cores": 1,
                             "elems_per_s": round(n1 / t1, 1), "seconds": round(t1, 1)}}
+
+
+GROUP_ELEMS = 1 << 27   # elements per node copied to the host at a time (full baselines)
+
+
+def _host_slot(ptr, n, dtype):
+    """Host copy of n stored elements at a device address (bf16 as uint16 words)."""
+    import numpy as np
+    from paper_2608_28670_gb300.runner import device_view
+    v = device_view(ptr, n, dtype).cpu().numpy()
+    return v.view(np.uint16) if v.dtype == np.int16 else v
+
+
+def cpu_baseline_full(run, min_seconds=0.5):
+    """The unmodified fp64 oracle over every element of the workload: each layer's forecast
+    from its live history slots (and on the sampler layer the Euler update), on one core and
+    on every core (spawned workers).  Layers are copied to the host in groups of about
+    GROUP_ELEMS elements per node outside the timed regions; only oracle calls are timed.  A
+    workload that takes less than `min_seconds` on one core is processed repeatedly."""
+    import numpy as np
+    import oracle
+    p = run.problem
+    W = oracle.paper_weights(list(p.nodes), p.t)
+    m = len(p.nodes)
+    slots = [bc_slot_ptrs(run, j) for j in range(m)]
+    groups, cur, n_cur = [], [], 0
+    for l in range(run.n_feat):
+        n = run.numels[l]
+        if cur and n_cur + n > GROUP_ELEMS:
+            groups.append(cur)
+            cur, n_cur = [], 0
+        cur.append(l)
+        n_cur += n
+    if cur:
+        groups.append(cur)
+    cap = max(sum(run.numels[l] for l in g) for g in groups)
+    one_s = all_s = 0.0
+    elems = 0
+    pool = None
+    passes = 1
+    try:
+        for gi, g in enumerate(groups):
+            F = [np.concatenate([_host_slot(slots[j][l], run.numels[l], run.w.dtype)
+                                 for l in g]) for j in range(m)]
+            chunks = [[f[o:o + CHUNK] for f in F] for o in range(0, F[0].size, CHUNK)]
+            if gi == 0:
+                t0 = time.perf_counter()
+                for c in chunks:
+                    oracle.combine(c, W)
+                first = time.perf_counter() - t0
+                if len(groups) == 1 and first < min_seconds:
+                    passes = max(1, int(min_seconds / max(first, 1e-6)))
+            t0 = time.perf_counter()
+            for _ in range(passes):
+                for c in chunks:
+                    oracle.combine(c, W)
+            one_s += time.perf_counter() - t0
+            if pool is None:
+                pool = OraclePool(F, W, capacity=cap)
+            else:
+                pool.load(F)
+            _, secs = pool.run(passes)
+            all_s += secs
+            elems += F[0].size
+            del F, chunks
+        if run.euler:
+            l = len(run.numels) - 1
+            V = [_host_slot(slots[j][l], run.numels[l], run.w.dtype) for j in range(m)]
+            x = run.x.cpu().numpy()
+            t0 = time.perf_counter()
+            for _ in range(passes):
+                oracle.euler(V, W, x, p.dt)
+            te = time.perf_counter() - t0
+            one_s += te
+            all_s += te
+            elems += V[0].size
+        cores = pool.workers
+    finally:
+        if pool is not None:
+            pool.close()
+    alg = run.algorithmic_bytes() * passes
+    return {"value": round(alg / all_s / 1e9, 4), "unit": "GB/s", "cores": cores,
+            "kind": "oracle", "elems_per_s": round(elems * passes / all_s, 1),
+            "seconds": round(all_s, 3),
+            "sample": f"the whole workload: {elems} elements ({run.n_feat} layers"
+                      f"{' + the Euler layer' if run.euler else ''}, K={m}), "
+                      f"{passes} pass(es), fp64 oracle on {cores} spawned workers"
+                      f"{'; the Euler layer on one core' if run.euler else ''}",
+            "single_core": {"value": round(alg / one_s / 1e9, 4), "cores": 1,
+                            "elems_per_s": round(elems * passes / one_s, 1),
+                            "seconds": round(one_s, 3)}}
 
 
 def bc_slot_ptrs(run, j):

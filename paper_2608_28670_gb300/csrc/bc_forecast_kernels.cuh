@@ -55,13 +55,19 @@
 #define BC_TMA_STAGES 3
 #endif
 #ifndef BC_TMA_VPT_K4
-#define BC_TMA_VPT_K4 2
+#define BC_TMA_VPT_K4 1      // 8 KiB tiles per history slot at H = 4
 #endif
 #ifndef BC_TMA_STAGES_K4
-#define BC_TMA_STAGES_K4 3   // 3 x 4 x 16 KiB = 192 KiB of shared memory
+#define BC_TMA_STAGES_K4 5   // 5 x 4 x 8 KiB = 160 KiB of shared memory
 #endif
 #ifndef BC_TMA_AUTO_K4
-#define BC_TMA_AUTO_K4 0     // 1: AUTO also picks the pipeline at H = 4 for large launches
+#define BC_TMA_AUTO_K4 1     // AUTO picks the pipeline at H = 4 for large launches too
+#endif
+#ifndef BC_TMA_MIN_TILES_PER_LAYER
+// AUTO runs the pipeline only when layers average at least this many of its tiles: many
+// small tensors (the blockwise layout: 4096 x 64 Ki bf16, eight 16 KiB tiles each) stream
+// faster through the register kernel (7.14 vs 7.00 TB/s at H = 3).
+#define BC_TMA_MIN_TILES_PER_LAYER 32
 #endif
 #ifndef BC_SMALL_LAUNCH_TILES_PER_SM
 #define BC_SMALL_LAUNCH_TILES_PER_SM 2  // register launches below this many tiles per SM use VPT 1
@@ -301,6 +307,21 @@ __device__ __forceinline__ void seek_layer(const ForecastArgs<CAP> &a, int64_t t
     }
 }
 
+// The layer cursor of a CTA's first tile: from the host-computed starts when the launch has
+// them, else by binary search.
+template <int CAP>
+__device__ __forceinline__ void cta_first_layer(const ForecastArgs<CAP> &a, int64_t t_lo, int &l,
+                                                int64_t &first) {
+    if constexpr (CAP == 0) {
+        if (static_cast<int>(blockIdx.x) < a.n_starts) {
+            l = a.start[blockIdx.x].layer;
+            first = a.start[blockIdx.x].first;
+            return;
+        }
+    }
+    find_layer(a, t_lo, l, first);
+}
+
 // Forecast one history vector from its K raw pieces (node order j = 1..K), store it, and
 // on the update layer apply x <- ca x + cb v_hat (+ cc z) to the same elements.
 template <int K, class TIn, class TOut, int CAP>
@@ -416,10 +437,13 @@ __global__ void __launch_bounds__(kThreads)
     if (t_lo >= t_hi) return;
     int l;
     int64_t first;
-    find_layer(a, t_lo, l, first);
+    cta_first_layer(a, t_lo, l, first);
+    LayerEntry L = entry_of(a, l);
     for (int64_t tile = t_lo; tile < t_hi; ++tile) {
-        seek_layer(a, tile, l, first);
-        const LayerEntry L = entry_of(a, l);
+        if (tile >= L.tile_end) {
+            seek_layer(a, tile, l, first);
+            L = entry_of(a, l);
+        }
         const int64_t nvec = L.numel / (kVecBytes / TIn::kBytes);
         const int64_t v0 = (tile - first) * kTileVecs + threadIdx.x;
         const char *src[K];
@@ -473,8 +497,6 @@ template <int K>
 constexpr int kTmaTileBytes = kThreads * kTmaVpt<K> * kVecBytes;
 template <int K>
 constexpr int kTmaSmemBytes = kTmaStages<K> * K * kTmaTileBytes<K>;
-static_assert(kTmaSmemBytes<4> <= 227 * 1024, "H = 4 ring exceeds shared memory");
-static_assert(kTmaSmemBytes<3> <= 227 * 1024, "H = 3 ring exceeds shared memory");
 
 template <int K, class TIn, class TOut, int CAP>
 __global__ void __launch_bounds__(kThreads)
@@ -484,8 +506,25 @@ __global__ void __launch_bounds__(kThreads)
     constexpr int kTileBytes = kTmaTileBytes<K>;
     constexpr int EV = kVecBytes / TIn::kBytes;
     constexpr int S = kTmaStages<K>;
+    static_assert(kTmaSmemBytes<K> <= 227 * 1024, "the ring exceeds a CTA's shared memory");
     extern __shared__ __align__(128) unsigned char stage_mem[];
     __shared__ __align__(8) uint64_t full[S];
+    // kMeta: the producer hands each stage's layer (entry, index, first tile) to the consumers
+    // through shared memory, written before the stage is armed and read after the wait (the
+    // mbarrier arrival releases it), so the consumers never touch the layer table.  That pays
+    // where the table is in device memory; with the parameter-block table it measured +0.5 %
+    // at H = 3 and -1.2 % at H = 4 (-0.2 % at H = 2) on the video workload, so elsewhere the
+    // consumers keep their own cursor over the parameter block.
+    constexpr bool kMeta = CAP == 0 || K == 3;
+    // kCache: producer and consumers keep the current layer's entry in registers and re-read
+    // the table only on crossing into the next layer.  Measured on the video workload against
+    // re-reading the parameter-block entry on every tile: +0.5 % at H = 2, -2 % at H = 4
+    // (8 KiB tiles, five stages; reproducible on two boxes, cause not isolated), so H = 4
+    // re-reads per tile unless the table is in device memory.
+    constexpr bool kCache = CAP == 0 || K != 4;
+    __shared__ LayerEntry stage_entry[kMeta ? S : 1];
+    __shared__ int32_t stage_layer[kMeta ? S : 1];
+    __shared__ int64_t stage_first[kMeta ? S : 1];
     __shared__ int abort_flag;
 
     float w[K];
@@ -506,9 +545,18 @@ __global__ void __launch_bounds__(kThreads)
     int pl = 0;
     int64_t pfirst = 0;
     int64_t issued = 0;
+    LayerEntry PL{};
     auto issue = [&](int64_t tile, int stage) {
-        seek_layer(a, tile, pl, pfirst);
-        const LayerEntry L = entry_of(a, pl);
+        if (!kCache || tile >= PL.tile_end) {
+            seek_layer(a, tile, pl, pfirst);
+            PL = entry_of(a, pl);
+        }
+        const LayerEntry &L = PL;
+        if constexpr (kMeta) {
+            stage_entry[stage] = L;
+            stage_layer[stage] = pl;
+            stage_first[stage] = pfirst;
+        }
         const int64_t nvec = L.numel / EV;
         const int64_t v_first = (tile - pfirst) * kTileVecs;
         int64_t nv = nvec - v_first;
@@ -528,13 +576,18 @@ __global__ void __launch_bounds__(kThreads)
         ++issued;
     };
     if (threadIdx.x == 0 && t_lo < t_hi) {
-        find_layer(a, t_lo, pl, pfirst);
+        cta_first_layer(a, t_lo, pl, pfirst);
+        PL = entry_of(a, pl);
         for (int i = 0; i < S && t_lo + i < t_hi; ++i) issue(t_lo + i, i);
     }
 
-    int l = 0;
+    int l = 0;                // the consumers' own cursor (without kMeta)
     int64_t first = 0;
-    if (t_lo < t_hi) find_layer(a, t_lo, l, first);
+    LayerEntry CL{};
+    if (!kMeta && t_lo < t_hi) {
+        cta_first_layer(a, t_lo, l, first);
+        CL = entry_of(a, l);
+    }
     for (int64_t tile = t_lo; tile < t_hi; ++tile) {
         const int64_t i = tile - t_lo;
         const int stage = static_cast<int>(i % S);
@@ -551,12 +604,26 @@ __global__ void __launch_bounds__(kThreads)
             }
             return;
         }
-        seek_layer(a, tile, l, first);
-        const LayerEntry L = entry_of(a, l);
+        LayerEntry L;
+        int64_t lfirst;
+        int lidx;
+        if constexpr (kMeta) {
+            L = stage_entry[stage];
+            lfirst = stage_first[stage];
+            lidx = stage_layer[stage];
+        } else {
+            if (!kCache || tile >= CL.tile_end) {
+                seek_layer(a, tile, l, first);
+                CL = entry_of(a, l);
+            }
+            L = CL;
+            lfirst = first;
+            lidx = l;
+        }
         const int64_t nvec = L.numel / EV;
-        const int64_t v0 = (tile - first) * kTileVecs;
+        const int64_t v0 = (tile - lfirst) * kTileVecs;
         char *dst = reinterpret_cast<char *>(L.dst);
-        const bool euler = (l == a.euler_layer);
+        const bool euler = (lidx == a.euler_layer);
         const unsigned char *sb = stage_mem + static_cast<size_t>(stage) * K * kTileBytes;
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
@@ -699,9 +766,11 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
     constexpr int kRegVpt = kVecsPerThreadFor<K>;
     const bool pipe_ok = K <= 3 || BC_TMA_AUTO_K4;
     bool pipeline = p.kernel == BC_KERNEL_PIPELINE || p.inject;
-    if (!pipeline && p.kernel == BC_KERNEL_AUTO && pipe_ok)
-        pipeline = count_tiles(layers, n, TIn::kBytes, kThreads * kTmaVpt<K>) >=
-                   static_cast<int64_t>(kTmaMinTilesPerCta) * sms;
+    if (!pipeline && p.kernel == BC_KERNEL_AUTO && pipe_ok) {
+        const int64_t tiles = count_tiles(layers, n, TIn::kBytes, kThreads * kTmaVpt<K>);
+        pipeline = tiles >= static_cast<int64_t>(kTmaMinTilesPerCta) * sms &&
+                   tiles >= static_cast<int64_t>(BC_TMA_MIN_TILES_PER_LAYER) * n;
+    }
     int vpt = kRegVpt;
     if (!pipeline && CAP == kLayersSmall && p.kernel == BC_KERNEL_AUTO && kRegVpt > 1 &&
         count_tiles(layers, n, TIn::kBytes, kThreads * kRegVpt) <
@@ -717,6 +786,26 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         const int err = upload_table(*p.table, tab.data(), n, s);
         if (err != cudaSuccess) return err;
         a.table = p.table->dev;
+        // every CTA's first layer, as the kernels would find it (grid as launched below)
+        int64_t grid_cap = sms;
+        if (!pipeline) {
+            static std::atomic<int> occ_reg{0};
+            grid_cap *= resident_ctas(forecast_kernel<K, kRegVpt, TIn, TOut, 0>, occ_reg,
+                                      BC_CTAS_PER_SM);
+        }
+        const int64_t grid = a.total_tiles < grid_cap ? a.total_tiles : grid_cap;
+        const int64_t per_cta = (a.total_tiles + grid - 1) / grid;
+        a.n_starts = 0;
+        if (grid <= kMaxStartCtas) {
+            int l = 0;
+            for (int64_t c = 0; c < grid; ++c) {
+                const int64_t t = c * per_cta;
+                while (l < n - 1 && t >= tab[l].tile_end) ++l;
+                a.start[c].layer = l;
+                a.start[c].first = l > 0 ? tab[l - 1].tile_end : 0;
+            }
+            a.n_starts = static_cast<int32_t>(grid);
+        }
     } else {
         a.total_tiles = fill_entries(a.layer, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
         if (a.total_tiles == 0) return cudaSuccess;

@@ -61,6 +61,16 @@ struct LayerEntry {        // 32 bytes
     int64_t tile_end;      // exclusive prefix sum of tiles up to this layer
 };
 
+// Where a CTA's contiguous tile range starts: the layer holding its first tile and that
+// layer's first tile.  Computed by the host for launches whose table is in device memory, so
+// that no CTA starts with a binary search of dependent global loads.
+struct CtaStart {
+    int64_t first;         // first tile of `layer`
+    int32_t layer;
+    int32_t pad;
+};
+constexpr int kMaxStartCtas = 512;
+
 template <int CAP>
 struct ForecastArgs {
     uint64_t slot[BC_MAX_K];  // slot base address of node j (j = 0 newest)
@@ -76,6 +86,8 @@ struct ForecastArgs {
     int32_t inject;           // test hook: leave the first pipeline stage unarmed
     int64_t total_tiles;
     const LayerEntry *table;  // CAP == 0: the layer table in device memory
+    int32_t n_starts;         // CAP == 0: CTAs whose first layer is given in `start`
+    CtaStart start[CAP > 0 ? 1 : kMaxStartCtas];  // CAP == 0: layer of each CTA's first tile
     LayerEntry layer[CAP > 0 ? CAP : 1];  // CAP > 0: the layer table itself
 };
 
