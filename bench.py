@@ -63,6 +63,9 @@ def parse_args():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-extra", action="store_true",
                     help="skip the push and fused-step measurements")
+    ap.add_argument("--warmup-min-s", type=float, default=None,
+                    help="least wall time of every leg's warm-up (default 0.25 s; profiling "
+                         "runs under ncu may shorten it)")
     ap.add_argument("--kernel", choices=["auto", "register", "pipeline"], default="auto",
                     help="pin the forecast kernel of the headline leg (default: the library's "
                          "choice)")
@@ -241,10 +244,11 @@ def window_targets(w, K):
     return ts or [rep.t]
 
 
-def warm_up(step, count, min_s=MIN_WARMUP_S):
+def warm_up(step, count, min_s=None):
     """Run `step(i)` at least `count` times and for at least `min_s` seconds of wall time
-    (synchronised); returns the number of steps run."""
+    (default MIN_WARMUP_S; synchronised); returns the number of steps run."""
     import torch
+    min_s = MIN_WARMUP_S if min_s is None else min_s
     t0 = time.perf_counter()
     i = 0
     while i < count:
@@ -304,6 +308,9 @@ def time_forecast(run, steps, warmup, stream, dist=None):
 
 
 def run_ours(args):
+    global MIN_WARMUP_S
+    if args.warmup_min_s is not None:
+        MIN_WARMUP_S = max(0.0, args.warmup_min_s)
     import torch
     from paper_2608_28670_gb300 import barycache as bc
     from paper_2608_28670_gb300.configs import WORKLOADS, T2V_HBM_BUDGET
