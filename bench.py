@@ -100,18 +100,24 @@ def _code_only(src: bytes) -> bytes:
     return re.sub(r"\s+", "", text).encode()
 
 
-def kernel_source_hash() -> str:
-    """Hash of the forecast kernels' device code (bc_forecast_kernels.cuh up to its host
-    launch plumbing, the tuning macros included) and of the headers it includes from the
-    package (layout, pipeline primitives), comments and whitespace ignored: a change there
-    voids a stored ncu figure."""
+HOST_SIDE_START = "// ------------------------------------------------------------------ host side"
+
+
+def kernel_source_hash(root: str = ROOT) -> str:
+    """Hash of the forecast kernels' device code: bc_forecast_kernels.cuh up to its host
+    launch plumbing (the tuning macros included), the kernel-visible part of bc_internal.h
+    (layout, tiling, launch arguments; up to its host-side marker) and the pipeline
+    primitives of bc_tma.cuh, comments and whitespace ignored.  A change there voids a stored
+    ncu figure; host-side plumbing does not."""
     h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2608_28670_gb300", "csrc")
-    with open(os.path.join(csrc, "bc_forecast_kernels.cuh"), "rb") as fh:
-        h.update(_code_only(fh.read().split(KERNEL_CODE_END.encode(), 1)[0]))
-    for name in ("bc_internal.h", "bc_tma.cuh"):
+    csrc = os.path.join(root, "paper_2608_28670_gb300", "csrc")
+    for name, marker in (("bc_forecast_kernels.cuh", KERNEL_CODE_END),
+                         ("bc_internal.h", HOST_SIDE_START), ("bc_tma.cuh", None)):
         with open(os.path.join(csrc, name), "rb") as fh:
-            h.update(_code_only(fh.read()))
+            text = fh.read()
+        if marker is not None:
+            text = text.split(marker.encode(), 1)[0]
+        h.update(_code_only(text))
     return h.hexdigest()[:16]
 
 
@@ -753,6 +759,18 @@ def time_blockwise(stream, steps):
         per_layer_launches = timed.launches
         st = bc.bc_cache_stats(h)
         ms_flat = timed(lambda: bc.bc_forecast_flat(h, 0.75, flat.data_ptr(), stream))
+        flat_launches = timed.launches
+        # the full step of a blockwise cache: push every tensor (from the forecast's buffers)
+        push_t = [0.7 - 1e-4 * i for i in range(100000)]
+        k = [0]
+
+        def push():
+            bc.bc_cache_push(h, per, push_t[k[0]], stream)
+            k[0] += 1
+        bc.bc_cache_set_kernel(h, bc.KERNEL_AUTO)
+        ms_push = timed(push)
+        push_launches = timed.launches
+        push_bytes = 2 * 2 * n * n_t
         return {"tensors": n_t, "elements_per_tensor": n,
                 "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
                               "ms": round(ms_layers, 4),
@@ -760,7 +778,12 @@ def time_blockwise(stream, steps):
                               "table_uploads": st["table_uploads"],
                               "GB/s_by_kernel": by_kernel},
                 "flat": {"GB/s": round(alg / (ms_flat * 1e-3) / 1e9, 1), "ms": round(ms_flat, 4),
-                         "launches_per_call": timed.launches}}
+                         "launches_per_call": flat_launches},
+                "push": {"GB/s": round(push_bytes / (ms_push * 1e-3) / 1e9, 1),
+                         "ms": round(ms_push, 4), "launches_per_call": push_launches,
+                         "bytes_per_push": push_bytes,
+                         "table_uploads": bc.bc_cache_stats(h)["table_uploads"]
+                                          - st["table_uploads"]}}
     finally:
         bc.bc_cache_destroy(h)
 

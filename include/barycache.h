@@ -25,11 +25,12 @@
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  All
  *    device work is enqueued on it asynchronously; errors are reported by return value
  *    only, and no call blocks on the device except bc_cache_create/destroy and
- *    bc_cache_check.
+ *    bc_cache_check (and a forecast or push over more than 1016 layers with a new layer
+ *    table while four earlier uploads are still queued; see bc_forecast).
  *  - CUDA graphs: while `stream` is being captured, pushes, commits, forecasts (all
  *    variants) and the probe drift enqueue kernels only (no allocation, copy or
- *    synchronisation), so they may be called during capture (outside capture, a forecast
- *    over more than 1016 layers may also copy its layer table to the device).  The graph holds the slot addresses, weights and update
+ *    synchronisation), so they may be called during capture (outside capture, a forecast or
+ *    push over more than 1016 layers may also copy its layer table to the device).  The graph holds the slot addresses, weights and update
  *    coefficients chosen when each call was made; replaying it repeats that device work
  *    and does not move the handle's host state (ring head, node times, statistics).  The
  *    first forecast of each kind on a device also queries and sets per-device kernel
@@ -114,7 +115,8 @@ typedef struct {
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
     int64_t pipeline_launches; /* of kernel_launches: TMA pipeline kernels (any call) */
-    int64_t table_uploads;   /* device layer-table uploads (forecasts of > 1016 layers) */
+    int64_t table_uploads;   /* device layer-table uploads (forecasts and pushes of > 1016
+                                layers) */
 } bc_stats;
 
 /* ---------------------------------------------------------------- host-only calls */
@@ -151,9 +153,10 @@ bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtyp
 /* Create the cache context H_t of Eq. 6 for `n_layers` tensors of numels[l] elements of
  * `dtype`, with history length K (1..BC_MAX_K).  Allocates, on the current device, one
  * arena of bc_cache_bytes_for(...) bytes and 16 KiB of reduction scratch for
- * bc_probe_drift plus a status word, and for caches of more than 1016 layers a layer table
- * of 32 bytes per layer in device memory and the same in pinned host memory (the only
- * allocations the library makes; freed by bc_cache_destroy).  p == NULL uses the paper's
+ * bc_probe_drift plus a status word, and for caches of more than 1016 layers two layer
+ * tables (forecast, push) of 32 bytes per layer in device memory, each with four times that
+ * of pinned host staging (the only allocations the library makes; freed by
+ * bc_cache_destroy).  p == NULL uses the paper's
  * defaults.  Blocks until the allocation is done.  Errors: INVALID_ARG, OOM, CUDA. */
 bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
                           const bc_params *p, bc_handle *out);
@@ -184,7 +187,10 @@ bc_status bc_cache_reset(bc_handle h);
  * head, and layer_ptrs[l] (device, numels[l] elements of the cache dtype, 16-byte
  * aligned) is copied into it by one grouped, byte-exact copy kernel on `stream`: with
  * AUTO, TMA bulk copies through a three-stage shared-memory ring (one warp per SM) once the
- * push has at least 16 tiles of 32 KiB per SM, else register loads and stores.  The node
+ * push has at least 16 tiles of 32 KiB per SM, else register loads and stores.  Beyond 1016
+ * layers the launch reads its layer table from the handle's device copy, re-uploaded only
+ * when the sources differ from the previous push (outside stream capture; while `stream` is
+ * captured, one launch per 1016 layers).  The node
  * counts as pushed when the call returns; if the pipeline copy gives up waiting (reported
  * by bc_cache_check) the slot's contents are undefined and the cache should be reset.  `t`
  * is the timestep of this full step.  Errors: INVALID_ARG (null pointer, non-finite t,
@@ -225,8 +231,10 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  * One persistent grouped kernel launch covers every selected layer.  Beyond 1016 selected
  * layers the launch reads its layer table from the handle's device copy, which is
  * re-uploaded (one cudaMemcpyAsync on `stream`, from pinned memory) only when the outputs
- * differ from the previous such call; while `stream` is being captured into a CUDA graph it
- * issues one launch per 1016 layers instead, so that the graph holds its own tables.
+ * differ from the previous such call; the host waits only if four uploads of different
+ * tables are still queued ahead of the device.  While `stream` is being captured into a CUDA
+ * graph it issues one launch per 1016 layers instead, so that the graph holds its own
+ * tables.
  * Layers with a NULL output are skipped, which also serves to forecast a window of layers.
  * Outputs must not overlap the arena (checked) or each other (not checked: overlapping
  * outputs race).

@@ -2,7 +2,7 @@
 // features in the evicted slot) and the dispatch of the forecast by history length.
 //
 // Both copy kernels walk the same kind of layer table as the forecast (carried in the launch's
-// parameter block, up to kLayersLarge layers per launch):
+// parameter block, or for more than kLayersLarge layers in the handle's device table):
 //   copy_tma_kernel  TMA bulk loads and stores through a three-stage shared-memory ring, one
 //                    warp per SM (large pushes);
 //   copy_kernel      16-byte register loads and stores at full occupancy (small pushes).
@@ -14,7 +14,7 @@
 namespace bc {
 namespace {
 
-// Grouped byte-exact copy for the push: layer.src -> layer.dst, numel elements of T.
+// Grouped byte-exact copy for the push: layer.src -> slot[0] + layer.dst, numel elements of T.
 // Always 16-byte vectors: the caller's source is only guaranteed 16-byte alignment.
 template <class T, int CAP>
 __global__ void __launch_bounds__(kThreads) copy_kernel(const __grid_constant__ ForecastArgs<CAP> a) {
@@ -24,13 +24,23 @@ __global__ void __launch_bounds__(kThreads) copy_kernel(const __grid_constant__ 
     int l = 0;
     int64_t first = 0;
     if (blockIdx.x < a.total_tiles) find_layer(a, blockIdx.x, l, first);
+    LayerEntry L = entry_of(a, l);
     for (int64_t tile = blockIdx.x; tile < a.total_tiles; tile += gridDim.x) {
-        seek_layer(a, tile, l, first);
-        const LayerEntry &L = a.layer[l];
+        if constexpr (CAP == 0) {
+            // device-memory table: a grid stride may cross many small layers, so search
+            // instead of stepping through every entry
+            if (tile >= L.tile_end) {
+                find_layer(a, tile, l, first);
+                L = entry_of(a, l);
+            }
+        } else {
+            seek_layer(a, tile, l, first);
+            L = a.layer[l];
+        }
         const int64_t nvec = L.numel / EV;
         const int64_t v0 = (tile - first) * kTileVecs + threadIdx.x;
         const char *src = reinterpret_cast<const char *>(L.src);
-        char *dst = reinterpret_cast<char *>(L.dst);
+        char *dst = reinterpret_cast<char *>(a.slot[0] + L.dst);
         uint4 r[kVecsPerThread];
 #pragma unroll
         for (int u = 0; u < kVecsPerThread; ++u) {
@@ -98,11 +108,15 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
 
     int pl;                   // lane 0's load cursor
     int64_t pfirst;
-    find_layer(a, t_lo, pl, pfirst);
+    cta_first_layer(a, t_lo, pl, pfirst);
+    LayerEntry PL = entry_of(a, pl);
     int64_t issued = 0;
     auto issue = [&](int64_t tile, int stage) {
-        seek_layer(a, tile, pl, pfirst);
-        const LayerEntry &L = a.layer[pl];
+        if (CAP > 0 || tile >= PL.tile_end) {
+            seek_layer(a, tile, pl, pfirst);
+            PL = entry_of(a, pl);
+        }
+        const LayerEntry &L = PL;
         const int64_t g0 = (tile - pfirst) * kTileGroups;
         int64_t ng = L.numel / EV - g0;
         ng = ng > kTileGroups ? kTileGroups : (ng < 0 ? 0 : ng);
@@ -122,7 +136,8 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
 
     int l;                    // every lane's store cursor
     int64_t first;
-    find_layer(a, t_lo, l, first);
+    cta_first_layer(a, t_lo, l, first);
+    LayerEntry L = entry_of(a, l);
     for (int64_t tile = t_lo; tile < t_hi; ++tile) {
         const int64_t i = tile - t_lo;
         const int stage = static_cast<int>(i % S);
@@ -140,8 +155,10 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
             }
             return;
         }
-        seek_layer(a, tile, l, first);
-        const LayerEntry &L = a.layer[l];
+        if (CAP > 0 || tile >= L.tile_end) {
+            seek_layer(a, tile, l, first);
+            L = entry_of(a, l);
+        }
         const int64_t nvec = L.numel / EV;
         if (lane == 0) {
             const int64_t g0 = (tile - first) * kTileGroups;
@@ -149,7 +166,7 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
             ng = ng > kTileGroups ? kTileGroups : (ng < 0 ? 0 : ng);
             if (ng > 0) {
                 fence_proxy_async_shared();
-                bulk_store_from_shared(reinterpret_cast<char *>(L.dst) + g0 * 16,
+                bulk_store_from_shared(reinterpret_cast<char *>(a.slot[0] + L.dst) + g0 * 16,
                                        stage_mem + static_cast<size_t>(stage) * kCopyTileBytes,
                                        static_cast<uint32_t>(ng * 16));
             }
@@ -163,7 +180,7 @@ __global__ void __launch_bounds__(kCopyTmaThreads)
         if (rem != 0 && tile == L.tile_end - 1 && lane < rem) {
             const int64_t e = nvec * EV + lane;
             using St = typename T::store_t;
-            reinterpret_cast<St *>(L.dst)[e] = reinterpret_cast<const St *>(L.src)[e];
+            reinterpret_cast<St *>(a.slot[0] + L.dst)[e] = reinterpret_cast<const St *>(L.src)[e];
         }
     }
     if (lane == 0) bulk_wait_group_all();
@@ -178,29 +195,46 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
     a.euler_layer = -1;
     a.status = opt.status;
     a.inject = opt.inject;
+    a.slot[0] = opt.dst_base;
     // The bulk-copy pipeline needs enough of its 32 KiB tiles per SM to amortise its ring.
     a.n_layers = n;
-    a.total_tiles = fill_entries(a.layer, layers, n, T::kBytes, 16, kCopyTileBytes / 16);
-    if (a.total_tiles == 0) return cudaSuccess;
+    const int sms = sm_count();
     const bool pipeline =
         opt.kernel == BC_KERNEL_PIPELINE || opt.inject ||
         (opt.kernel == BC_KERNEL_AUTO &&
-         a.total_tiles >= static_cast<int64_t>(kCopyMinTilesPerCta) * sm_count());
+         count_tiles(layers, n, T::kBytes, kCopyTileBytes / kVecBytes) >=
+             static_cast<int64_t>(kCopyMinTilesPerCta) * sms);
+    const int tile_groups = pipeline ? kCopyTileBytes / 16 : kThreads * kCopyVecsPerThread;
+    if constexpr (CAP == 0) {
+        std::vector<LayerEntry> &tab = table_scratch();
+        tab.resize(static_cast<size_t>(n));
+        a.total_tiles = fill_entries(tab.data(), layers, n, T::kBytes, 16, tile_groups);
+        if (a.total_tiles == 0) return cudaSuccess;
+        const int err = upload_table(*opt.table, tab.data(), n, s);
+        if (err != cudaSuccess) return err;
+        a.table = opt.table->dev;
+        if (pipeline) {
+            const int64_t cap = static_cast<int64_t>(sms) * BC_COPY_CTAS_PER_SM;
+            fill_starts(a, tab.data(), n, a.total_tiles < cap ? a.total_tiles : cap);
+        }
+    } else {
+        a.total_tiles = fill_entries(a.layer, layers, n, T::kBytes, 16, tile_groups);
+        if (a.total_tiles == 0) return cudaSuccess;
+    }
     if (pipeline) {
         auto kern = copy_tma_kernel<T, CAP>;
         static std::atomic<bool> attr_set[64];
         const int err = ensure_smem_attribute(kern, attr_set, kCopySmemBytes);
         if (err != cudaSuccess) return err;
-        const int64_t cap = static_cast<int64_t>(sm_count()) * BC_COPY_CTAS_PER_SM;
+        const int64_t cap = static_cast<int64_t>(sms) * BC_COPY_CTAS_PER_SM;
         const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
         kern<<<grid, kCopyTmaThreads, kCopySmemBytes, s>>>(a);
         ++*launches;
         ++*pipeline_launches;
         return cudaGetLastError();
     }
-    a.total_tiles = fill_entries(a.layer, layers, n, T::kBytes, 16, kThreads * kCopyVecsPerThread);
     auto kern = copy_kernel<T, CAP>;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * resident_ctas(kern, occ, 0);
+    const int64_t cap = static_cast<int64_t>(sms) * resident_ctas(kern, occ, 0);
     const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
     kern<<<grid, kThreads, 0, s>>>(a);
     ++*launches;
@@ -210,6 +244,8 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
 template <class T>
 int copy_all(const LayerEntry *layers, int n_layers, const CopyOptions &opt, cudaStream_t s,
              int64_t *launches, int64_t *pipe) {
+    if (n_layers > kLayersLarge && opt.table != nullptr && n_layers <= opt.table->capacity)
+        return copy_group<T, 0>(layers, n_layers, opt, s, launches, pipe);
     int err = cudaSuccess;
     for (int base = 0; base < n_layers && err == cudaSuccess; base += kLayersLarge) {
         const int n = n_layers - base < kLayersLarge ? n_layers - base : kLayersLarge;

@@ -709,26 +709,49 @@ inline int64_t fill_entries(LayerEntry *dst, const LayerEntry *layers, int n, in
 }
 
 // Make the handle's device table hold `entries[0..n)`: one cudaMemcpyAsync on `s` from the
-// pinned staging, skipped when the previous upload was the same table.  Before the staging
-// is overwritten, the previous upload's copy must have read it (its event).
+// next pinned staging buffer, skipped when the previous upload was the same table.  A staging
+// buffer is rewritten only after the copy that last read it has run (its event).
 inline int upload_table(DeviceTable &tb, const LayerEntry *entries, int n, cudaStream_t s) {
     const size_t bytes = sizeof(LayerEntry) * static_cast<size_t>(n);
-    if (tb.valid == n && std::memcmp(tb.host, entries, bytes) == 0) return cudaSuccess;
-    cudaEvent_t ev = static_cast<cudaEvent_t>(tb.uploaded);
-    if (tb.pending) {
+    if (tb.valid == n && tb.last >= 0 &&
+        std::memcmp(tb.host + static_cast<size_t>(tb.last) * tb.capacity, entries, bytes) == 0)
+        return cudaSuccess;
+    const int k = (tb.last + 1) % kTableStaging;
+    cudaEvent_t ev = static_cast<cudaEvent_t>(tb.uploaded[k]);
+    if (tb.pending[k]) {
         const cudaError_t e = cudaEventSynchronize(ev);
         if (e != cudaSuccess) return e;
+        tb.pending[k] = false;
     }
-    std::memcpy(tb.host, entries, bytes);
+    LayerEntry *stage = tb.host + static_cast<size_t>(k) * tb.capacity;
+    std::memcpy(stage, entries, bytes);
     tb.valid = 0;
-    cudaError_t e = cudaMemcpyAsync(tb.dev, tb.host, bytes, cudaMemcpyHostToDevice, s);
+    cudaError_t e = cudaMemcpyAsync(tb.dev, stage, bytes, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return e;
     e = cudaEventRecord(ev, s);
     if (e != cudaSuccess) return e;
-    tb.pending = true;
+    tb.pending[k] = true;
+    tb.last = k;
     tb.valid = n;
     ++tb.uploads;
     return cudaSuccess;
+}
+
+// Fill a.start[] with the layer of every CTA's first tile (contiguous ranges of
+// ceil(total / grid) tiles), as the kernels would find it.
+template <int CAP>
+inline void fill_starts(ForecastArgs<CAP> &a, const LayerEntry *tab, int n, int64_t grid) {
+    a.n_starts = 0;
+    if (grid > kMaxStartCtas || grid < 1) return;
+    const int64_t per_cta = (a.total_tiles + grid - 1) / grid;
+    int l = 0;
+    for (int64_t c = 0; c < grid; ++c) {
+        const int64_t t = c * per_cta;
+        while (l < n - 1 && t >= tab[l].tile_end) ++l;
+        a.start[c].layer = l;
+        a.start[c].first = l > 0 ? tab[l - 1].tile_end : 0;
+    }
+    a.n_starts = static_cast<int32_t>(grid);
 }
 
 // Host staging for the tile prefix sums of a device-table launch (one per host thread).
@@ -793,19 +816,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
             grid_cap *= resident_ctas(forecast_kernel<K, kRegVpt, TIn, TOut, 0>, occ_reg,
                                       BC_CTAS_PER_SM);
         }
-        const int64_t grid = a.total_tiles < grid_cap ? a.total_tiles : grid_cap;
-        const int64_t per_cta = (a.total_tiles + grid - 1) / grid;
-        a.n_starts = 0;
-        if (grid <= kMaxStartCtas) {
-            int l = 0;
-            for (int64_t c = 0; c < grid; ++c) {
-                const int64_t t = c * per_cta;
-                while (l < n - 1 && t >= tab[l].tile_end) ++l;
-                a.start[c].layer = l;
-                a.start[c].first = l > 0 ? tab[l - 1].tile_end : 0;
-            }
-            a.n_starts = static_cast<int32_t>(grid);
-        }
+        fill_starts(a, tab.data(), n, a.total_tiles < grid_cap ? a.total_tiles : grid_cap);
     } else {
         a.total_tiles = fill_entries(a.layer, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
         if (a.total_tiles == 0) return cudaSuccess;

@@ -214,7 +214,8 @@ struct bc_cache {
     Memo memo;
     bc_stats stats{};
     std::vector<bc::LayerEntry> scratch_entries;  // host staging for launch tables
-    bc::DeviceTable table;                        // device layer table (> 1016 layers only)
+    bc::DeviceTable table;                        // device layer tables (> 1016 layers only):
+    bc::DeviceTable push_table;                   //   forecasts, push copies
     double *probe_partials = nullptr;             // device scratch of bc_probe_drift
     uint32_t *status = nullptr;                   // device status word of the forecast kernels
     bool inject_next = false;                     // test hooks (bc_cache_inject_fault):
@@ -245,19 +246,21 @@ bc_status check_handle(bc_handle h) {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// The device layer table of a cache with more than kLayersLarge layers: n_layers entries of
-// device memory, the same of pinned host staging, and the event that orders reuse of the
-// staging after its last copy.
-bc_status alloc_table(bc_cache *h) {
-    bc::DeviceTable &tb = h->table;
-    const size_t bytes = sizeof(bc::LayerEntry) * static_cast<size_t>(h->n_layers);
+// A device layer table for a cache with more than kLayersLarge layers: n_layers entries of
+// device memory, kTableStaging times that of pinned host staging, and one event per staging
+// buffer that orders its reuse after the copy that last read it.
+bc_status alloc_table(bc::DeviceTable &tb, int n_layers) {
+    const size_t bytes = sizeof(bc::LayerEntry) * static_cast<size_t>(n_layers);
     void *dev = nullptr, *host = nullptr;
-    cudaEvent_t ev = nullptr;
+    cudaEvent_t ev[bc::kTableStaging] = {};
     cudaError_t e = cudaMalloc(&dev, bytes);
-    if (e == cudaSuccess) e = cudaHostAlloc(&host, bytes, cudaHostAllocDefault);
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaHostAlloc(&host, bytes * bc::kTableStaging, cudaHostAllocDefault);
+    for (int k = 0; k < bc::kTableStaging && e == cudaSuccess; ++k)
+        e = cudaEventCreateWithFlags(&ev[k], cudaEventDisableTiming);
     if (e != cudaSuccess) {
         cudaGetLastError();
+        for (int k = 0; k < bc::kTableStaging; ++k)
+            if (ev[k]) cudaEventDestroy(ev[k]);
         if (dev) cudaFree(dev);
         if (host) cudaFreeHost(host);
         return e == cudaErrorMemoryAllocation ? fail(BC_ERR_OOM, "layer table")
@@ -265,9 +268,28 @@ bc_status alloc_table(bc_cache *h) {
     }
     tb.dev = static_cast<bc::LayerEntry *>(dev);
     tb.host = static_cast<bc::LayerEntry *>(host);
-    tb.uploaded = ev;
-    tb.capacity = h->n_layers;
+    for (int k = 0; k < bc::kTableStaging; ++k) tb.uploaded[k] = ev[k];
+    tb.capacity = n_layers;
     return BC_OK;
+}
+
+bc_status alloc_table(bc_cache *h) {
+    bc_status s = alloc_table(h->table, h->n_layers);
+    if (s == BC_OK) s = alloc_table(h->push_table, h->n_layers);
+    return s;
+}
+
+cudaError_t free_table(bc::DeviceTable &tb) {
+    cudaError_t rc = cudaSuccess;
+    auto keep = [&rc](cudaError_t e) {
+        if (rc == cudaSuccess && e != cudaSuccess) rc = e;
+    };
+    if (tb.dev) keep(cudaFree(tb.dev));
+    if (tb.host) keep(cudaFreeHost(tb.host));
+    for (int k = 0; k < bc::kTableStaging; ++k)
+        if (tb.uploaded[k]) keep(cudaEventDestroy(static_cast<cudaEvent_t>(tb.uploaded[k])));
+    tb = bc::DeviceTable{};
+    return rc;
 }
 
 // Free every device and pinned allocation of the handle (the caller has synchronised).
@@ -278,12 +300,10 @@ cudaError_t free_device(bc_cache *h) {
     };
     if (h->arena) keep(cudaFree(h->arena));
     if (h->probe_partials) keep(cudaFree(h->probe_partials));
-    if (h->table.dev) keep(cudaFree(h->table.dev));
-    if (h->table.host) keep(cudaFreeHost(h->table.host));
-    if (h->table.uploaded) keep(cudaEventDestroy(static_cast<cudaEvent_t>(h->table.uploaded)));
+    keep(free_table(h->table));
+    keep(free_table(h->push_table));
     h->arena = nullptr;
     h->probe_partials = nullptr;
-    h->table = bc::DeviceTable{};
     return rc;
 }
 
@@ -331,15 +351,14 @@ bool ranges_overlap(uint64_t a, uint64_t an, uint64_t b, uint64_t bn) {
 // carry its tables in parameter blocks: few enough layers, no table on this handle, or a
 // stream that is being captured into a CUDA graph (a graph must hold every table it replays,
 // while the device table is rewritten by later calls).
-bc::DeviceTable *table_for(bc_cache *h, int n_layers, void *stream) {
-    if (n_layers <= bc::kLayersLarge || !h->table.dev || n_layers > h->table.capacity)
-        return nullptr;
+bc::DeviceTable *table_for(bc::DeviceTable &tb, int n_layers, void *stream) {
+    if (n_layers <= bc::kLayersLarge || !tb.dev || n_layers > tb.capacity) return nullptr;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     if (cudaStreamIsCapturing(static_cast<cudaStream_t>(stream), &cs) != cudaSuccess) {
         cudaGetLastError();
         return nullptr;
     }
-    return cs == cudaStreamCaptureStatusNone ? &h->table : nullptr;
+    return cs == cudaStreamCaptureStatusNone ? &tb : nullptr;
 }
 
 bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dtype out_dtype,
@@ -424,7 +443,7 @@ bc_status forecast_impl(bc_handle h, double t_new, void *const *out_ptrs, bc_dty
     if (plan.n_layers > 0) {
         DeviceGuard g(h->device);
         if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
-        plan.table = table_for(h, plan.n_layers, stream);
+        plan.table = table_for(h->table, plan.n_layers, stream);
         const int err = bc::launch_forecast(plan, stream, &h->stats.kernel_launches,
                                                 &h->stats.pipeline_launches);
         h->inject_next = false;
@@ -598,7 +617,7 @@ bc_status bc_cache_destroy(bc_handle h) {
     }
     h->magic = 0;
     bc_status rc = BC_OK;
-    if (h->arena || h->probe_partials || h->table.dev) {
+    if (h->arena || h->probe_partials || h->table.dev || h->push_table.dev) {
         DeviceGuard g(h->device);
         cudaError_t e = cudaDeviceSynchronize();
         if (e == cudaSuccess) e = free_device(h);
@@ -680,14 +699,17 @@ bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, vo
                 return fail(BC_ERR_INVALID_ARG, "layer %d source overlaps the cache arena", l);
             bc::LayerEntry e{};
             e.src = reinterpret_cast<uint64_t>(src);
-            e.dst = reinterpret_cast<uint64_t>(h->slot_base(next) + h->offset[l]);
+            e.dst = h->offset[l];
             e.numel = h->numel[l];
             entries.push_back(e);
         }
         if (!entries.empty()) {
             DeviceGuard g(h->device);
             if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
-            bc::CopyOptions opt{h->kernel, h->status, h->inject_next_push ? 1 : 0};
+            bc::CopyOptions opt{h->kernel, h->status, h->inject_next_push ? 1 : 0,
+                                table_for(h->push_table, static_cast<int>(entries.size()),
+                                          stream),
+                                reinterpret_cast<uint64_t>(h->slot_base(next))};
             const int err = bc::launch_copy(entries.data(), static_cast<int>(entries.size()),
                                             h->dtype, opt, stream, &h->stats.kernel_launches,
                                             &h->stats.pipeline_launches);
@@ -1020,7 +1042,7 @@ bc_status bc_cache_stats(bc_handle h, bc_stats *out) {
     if (!out) return fail(BC_ERR_INVALID_ARG, "out is NULL");
     h->stats.memo_hits = h->memo.hits;
     h->stats.memo_misses = h->memo.misses;
-    h->stats.table_uploads = h->table.uploads;
+    h->stats.table_uploads = h->table.uploads + h->push_table.uploads;
     *out = h->stats;
     return BC_OK;
 }

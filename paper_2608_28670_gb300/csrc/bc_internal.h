@@ -47,8 +47,8 @@ constexpr int kCopyVecsPerThread = 4;
 // small for the usual few-dozen-layer caches.  A forecast over more layers runs as one
 // launch that reads its table from a per-handle device copy (DeviceTable); while its stream
 // is being captured into a CUDA graph it issues one parameter-block launch per kLayersLarge
-// layers instead, so that the graph holds every table it replays.  Push copies of more than
-// kLayersLarge layers always issue one launch per group.
+// layers instead, so that the graph holds every table it replays.  Push copies work the same
+// way with a table of their own.
 constexpr int kLayersSmall = 8;
 constexpr int kLayersMedium = 64;
 constexpr int kLayersLarge = 1016;
@@ -56,7 +56,8 @@ constexpr int kLayersLarge = 1016;
 struct LayerEntry {        // 32 bytes
     uint64_t src;          // forecast: byte offset of the layer in every slot;
                            // copy: absolute source address
-    uint64_t dst;          // output address (forecast) / slot address (copy)
+    uint64_t dst;          // forecast: output address; copy: byte offset of the layer in
+                           // the destination slot (its base travels in the launch)
     int64_t numel;         // elements in the layer
     int64_t tile_end;      // exclusive prefix sum of tiles up to this layer
 };
@@ -94,18 +95,25 @@ struct ForecastArgs {
 // Kernel parameter blocks may hold up to 32,764 bytes (CUDA 12.1 and later).
 static_assert(sizeof(ForecastArgs<kLayersLarge>) <= 32764, "layer table exceeds the parameter block");
 
-// A device-memory copy of a launch's layer table, for forecasts over more layers than the
-// parameter block holds (one per handle; only caches of more than kLayersLarge layers have
-// one).  The table is uploaded from pinned staging with one cudaMemcpyAsync on the call's
-// stream, and only when it differs from the previous upload: a sampler that reuses its
-// output buffers uploads once.
+// ------------------------------------------------------------------ host side
+// (Everything below is the launchers' host-side view; the kernels see only what is above.)
+
+// A device-memory copy of a launch's layer table, for forecasts and pushes over more layers
+// than the parameter block holds (caches of more than kLayersLarge layers have one for each).
+// The table is uploaded with one cudaMemcpyAsync on the call's stream, and only when it
+// differs from the previous upload: a sampler that reuses its buffers uploads once.  The
+// pinned staging is a ring of kTableStaging buffers, each reused only after the copy that
+// last read it has run (its event), so the host waits only if that many uploads with
+// different tables are still queued ahead of the device.
+constexpr int kTableStaging = 4;
 struct DeviceTable {
     LayerEntry *dev = nullptr;     // device, `capacity` entries
-    LayerEntry *host = nullptr;    // pinned staging: the entries of the last upload
+    LayerEntry *host = nullptr;    // pinned staging: kTableStaging x `capacity` entries
     int capacity = 0;
     int valid = 0;                 // entries of the last upload (0: none yet)
-    bool pending = false;          // `uploaded` was recorded after an upload
-    void *uploaded = nullptr;      // cudaEvent_t recorded after the last upload
+    int last = -1;                 // staging buffer of the last upload
+    bool pending[kTableStaging] = {};        // an event was recorded after the buffer's copy
+    void *uploaded[kTableStaging] = {};      // cudaEvent_t per staging buffer
     int64_t uploads = 0;           // uploads so far
 };
 
@@ -204,13 +212,16 @@ int64_t static_drift_max_elems(bc_dtype dtype);
 int launch_drift_static(const void *cur, const void *prev, int64_t n, bc_dtype dtype,
                         double *out, void *stream, int64_t *launches);
 
-// Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst absolute):
+// Enqueue the grouped copy used by bc_cache_push (layers[].src absolute, .dst an offset in
+// the destination slot opt.dst_base):
 // the TMA bulk-copy pipeline for large pushes (or when pinned / injected), else the
 // register copy.  *pipeline_launches counts the former.
 struct CopyOptions {
     int kernel;               // bc_kernel
     uint32_t *status;         // device status word
     int inject;               // test hook: leave the pipeline's first stage unarmed
+    DeviceTable *table;       // non-null: more than kLayersLarge layers go in one launch
+    uint64_t dst_base;        // destination slot; layer l lands at dst_base + layers[l].dst
 };
 int launch_copy(const LayerEntry *layers, int n_layers, bc_dtype dtype, const CopyOptions &opt,
                 void *stream, int64_t *launches, int64_t *pipeline_launches);
