@@ -767,10 +767,14 @@ def time_blockwise(stream, steps):
         def push():
             bc.bc_cache_push(h, per, push_t[k[0]], stream)
             k[0] += 1
+        push_bytes = 2 * 2 * n * n_t
+        push_by_kernel = {}
+        for name, kern in (("register", bc.KERNEL_REGISTER), ("pipeline", bc.KERNEL_PIPELINE)):
+            bc.bc_cache_set_kernel(h, kern)
+            push_by_kernel[name] = round(push_bytes / (timed(push) * 1e-3) / 1e9, 1)
         bc.bc_cache_set_kernel(h, bc.KERNEL_AUTO)
         ms_push = timed(push)
         push_launches = timed.launches
-        push_bytes = 2 * 2 * n * n_t
         return {"tensors": n_t, "elements_per_tensor": n,
                 "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
                               "ms": round(ms_layers, 4),
@@ -781,6 +785,7 @@ def time_blockwise(stream, steps):
                          "launches_per_call": flat_launches},
                 "push": {"GB/s": round(push_bytes / (ms_push * 1e-3) / 1e9, 1),
                          "ms": round(ms_push, 4), "launches_per_call": push_launches,
+                         "GB/s_by_kernel": push_by_kernel,
                          "bytes_per_push": push_bytes,
                          "table_uploads": bc.bc_cache_stats(h)["table_uploads"]
                                           - st["table_uploads"]}}

@@ -158,10 +158,19 @@ def _ptr_array(ptrs):
     return (ctypes.c_void_p * len(ptrs))(*[p if p else None for p in ptrs])
 
 
+# Layer counts of the handles this module created (dropped when it destroys them), so that a
+# per-layer call does not pay an extra library round trip to learn the list length it must
+# check.  Handles created elsewhere are asked every time.
+_layer_counts: dict[int, int] = {}
+
+
 def _layer_count(h: int) -> int:
-    n = ctypes.c_int()
-    _check(lib().bc_cache_info(h, ctypes.byref(n), None, None), "bc_cache_info")
-    return n.value
+    n = _layer_counts.get(h)
+    if n is not None:
+        return n
+    c = ctypes.c_int()
+    _check(lib().bc_cache_info(h, ctypes.byref(c), None, None), "bc_cache_info")
+    return c.value
 
 
 def _layer_ptrs(h: int, ptrs: Sequence[int | None], where: str):
@@ -221,10 +230,12 @@ def bc_cache_create(numels: Sequence[int], K: int, dtype: int,
     _check(lib().bc_cache_create(arr, len(numels), K, dtype,
                                  ctypes.byref(params) if params else None, ctypes.byref(h)),
            "bc_cache_create")
+    _layer_counts[h.value] = len(numels)
     return h.value
 
 
 def bc_cache_destroy(h: int) -> None:
+    _layer_counts.pop(h, None)
     _check(lib().bc_cache_destroy(h), "bc_cache_destroy")
 
 

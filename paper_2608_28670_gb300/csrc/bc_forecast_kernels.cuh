@@ -652,6 +652,12 @@ __global__ void __launch_bounds__(kThreads)
 // several host threads at once, so these caches are atomics; threads that race to fill
 // one store the same value.
 
+// Pipeline CTAs per SM, each with its own ring (a launch-shape knob: two measured slower at
+// every H).
+#ifndef BC_TMA_CTAS_PER_SM
+#define BC_TMA_CTAS_PER_SM 1
+#endif
+
 // SM count of the current device, cached per device.
 inline int sm_count() {
     static std::atomic<int> cached[64];
@@ -810,7 +816,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         if (err != cudaSuccess) return err;
         a.table = p.table->dev;
         // every CTA's first layer, as the kernels would find it (grid as launched below)
-        int64_t grid_cap = sms;
+        int64_t grid_cap = static_cast<int64_t>(sms) * (pipeline ? BC_TMA_CTAS_PER_SM : 1);
         if (!pipeline) {
             static std::atomic<int> occ_reg{0};
             grid_cap *= resident_ctas(forecast_kernel<K, kRegVpt, TIn, TOut, 0>, occ_reg,
@@ -829,7 +835,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         static std::atomic<bool> attr_set[64];
         const int err = ensure_smem_attribute(kern, attr_set, smem);
         if (err != cudaSuccess) return err;
-        const int64_t cap = sms;
+        const int64_t cap = static_cast<int64_t>(sms) * BC_TMA_CTAS_PER_SM;
         const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
         kern<<<grid, kThreads, smem, s>>>(a);
         ++*launches;

@@ -168,6 +168,97 @@ static int device_checks(void) {
     return failures;
 }
 
+/* A blockwise-style cache of 2048 ragged bf16 tensors: pushes and the forecast each run as
+ * one launch (the layer tables travel through the handle's device copies), every element of
+ * every tensor matches the oracle, and a NaN planted in one stored value comes out as NaN. */
+static int many_layer_checks(void) {
+    enum { L = 2048 };
+    const double times[3] = {0.9, 0.85, 0.8};
+    const double t_new = 0.75;
+    static int64_t numels[L], offs[L + 1];
+    int64_t total = 0;
+    for (int l = 0; l < L; ++l) {
+        numels[l] = (l * 37) % 900 + 1 + (l % 9 == 0 ? 8192 : 0);
+        offs[l] = total;
+        total += (numels[l] + 7) / 8 * 8;       /* 16-byte aligned tensors in one buffer */
+    }
+    offs[L] = total;
+    uint16_t *host[3];
+    for (int k = 0; k < 3; ++k) {
+        host[k] = (uint16_t *)calloc((size_t)total, sizeof(uint16_t));
+        for (int l = 0; l < L; ++l)
+            for (int64_t e = 0; e < numels[l]; ++e) {
+                const double a = sin(0.01 * e + l), b = cos(0.003 * e - l);
+                host[k][offs[l] + e] = to_bf16((float)(a + b * times[k]));
+            }
+    }
+    const int64_t nan_layer = 777, nan_elem = 3;
+    host[1][offs[nan_layer] + nan_elem] = 0x7FC0;          /* NaN in the middle node */
+    void *dev_in = NULL, *dev_out = NULL;
+    bc_handle h = NULL;
+    CHECK(bc_cache_create(numels, L, 3, BC_DTYPE_BF16, NULL, &h) == BC_OK, "create: %s",
+          bc_last_error());
+    CHECK(cudaMalloc(&dev_in, (size_t)total * 2) == 0 && cudaMalloc(&dev_out, (size_t)total * 2) == 0,
+          "cudaMalloc");
+    static const void *src[L];
+    static void *outs[L];
+    for (int l = 0; l < L; ++l) {
+        src[l] = (const char *)dev_in + offs[l] * 2;
+        outs[l] = (char *)dev_out + offs[l] * 2;
+    }
+    bc_stats st0, st1;
+    CHECK(bc_cache_stats(h, &st0) == BC_OK, "stats");
+    for (int k = 0; k < 3 && !failures; ++k) {
+        CHECK(cudaMemcpy(dev_in, host[k], (size_t)total * 2, H2D) == 0, "upload");
+        CHECK(bc_cache_push(h, src, times[k], NULL) == BC_OK, "push: %s", bc_last_error());
+        cudaDeviceSynchronize();
+    }
+    CHECK(bc_forecast(h, t_new, outs, BC_DTYPE_BF16, NULL) == BC_OK, "forecast: %s",
+          bc_last_error());
+    CHECK(bc_cache_check(h) == BC_OK, "device status");
+    CHECK(bc_cache_stats(h, &st1) == BC_OK, "stats");
+    CHECK(st1.kernel_launches - st0.kernel_launches == 4, "%lld launches for 3 pushes and a "
+          "forecast of %d tensors", (long long)(st1.kernel_launches - st0.kernel_launches), L);
+    CHECK(st1.table_uploads - st0.table_uploads == 2, "%lld table uploads (one per table)",
+          (long long)(st1.table_uploads - st0.table_uploads));
+    uint16_t *got = (uint16_t *)malloc((size_t)total * 2);
+    CHECK(cudaMemcpy(got, dev_out, (size_t)total * 2, D2H) == 0, "download");
+    double nodes[3] = {times[2], times[1], times[0]}, W[3];
+    oracle_paper_weights(nodes, 3, t_new, 0.95, 0.0, 10.0, 1e-12, W);
+    double *ref = (double *)malloc((size_t)total * sizeof(double));
+    double *bound = (double *)malloc((size_t)total * sizeof(double));
+    int64_t bad = 0;
+    for (int l = 0; l < L; ++l) {
+        const void *F[3] = {host[2] + offs[l], host[1] + offs[l], host[0] + offs[l]};
+        oracle_combine(1, F, 3, W, numels[l], ref, bound);
+        for (int64_t e = 0; e < numels[l]; ++e) {
+            uint32_t u = (uint32_t)got[offs[l] + e] << 16;
+            float g;
+            memcpy(&g, &u, sizeof g);
+            if (isnan(ref[e])) {
+                if (!isnan(g)) ++bad;
+            } else if (!(fabs((double)g - ref[e]) <= ldexp(1.0, -8) * bound[e])) {
+                ++bad;
+            }
+        }
+        if (l == nan_layer) {
+            uint32_t u = (uint32_t)got[offs[l] + nan_elem] << 16;
+            float g;
+            memcpy(&g, &u, sizeof g);
+            CHECK(isnan(ref[nan_elem]) && isnan(g), "the planted NaN did not propagate");
+        }
+    }
+    CHECK(bad == 0, "%lld elements off the oracle", (long long)bad);
+    bc_cache_destroy(h);
+    cudaFree(dev_in);
+    cudaFree(dev_out);
+    for (int k = 0; k < 3; ++k) free(host[k]);
+    free(got);
+    free(ref);
+    free(bound);
+    return failures;
+}
+
 static double now_s(void) {
     struct timespec ts;
     clock_gettime(CLOCK_MONOTONIC, &ts);
@@ -224,6 +315,7 @@ int main(int argc, char **argv) {
     if (strcmp(argv[1], "host") == 0) rc = host_checks();
     else if (strcmp(argv[1], "device") == 0) rc = device_checks();
     else if (strcmp(argv[1], "hostcost") == 0) rc = host_cost();
+    else if (strcmp(argv[1], "manylayers") == 0) rc = many_layer_checks();
     else return 2;
     printf("%s checks: %s\n", argv[1], rc ? "FAILED" : "ok");
     return rc ? 1 : 0;

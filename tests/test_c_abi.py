@@ -39,6 +39,14 @@ def test_c_client_full_forecast_on_the_device(client):
 
 
 @pytest.mark.gpu
+def test_c_client_many_tensors_one_launch_each(client):
+    # 2048 tensors pushed and forecast from plain C: one launch per call, every element
+    # against the oracle, a planted NaN carried through
+    p = subprocess.run([client, "manylayers"], capture_output=True, text=True, timeout=300)
+    assert p.returncode == 0, p.stdout + p.stderr
+
+
+@pytest.mark.gpu
 def test_c_client_host_cost_mode_runs(client):
     # The timing mode reports one JSON line per cache size; the numbers are measurements,
     # so only their presence and sanity are checked here.
