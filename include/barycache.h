@@ -169,8 +169,9 @@ bc_status bc_cache_destroy(bc_handle h);
  * n_layers entries. */
 bc_status bc_cache_info(bc_handle h, int *n_layers, int *K, int *dtype);
 
-/* Device bytes held by this cache: the arena (the 16 KiB reduction scratch and host
- * bookkeeping are not counted). */
+/* Device bytes held by this cache: the arena, K slots of every layer at 256-byte aligned
+ * offsets (not counted: the 16 KiB reduction scratch and status word, the 32-byte-per-layer
+ * device layer tables of caches over 1016 layers, and host bookkeeping). */
 bc_status bc_cache_bytes(bc_handle h, int64_t *bytes);
 
 /* Replace the weight parameters (clears the weight memo). */
