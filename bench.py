@@ -501,7 +501,8 @@ def time_push(run, steps):
     from paper_2608_28670_gb300 import barycache as bc
     if run.window < run.n_feat or run.euler:
         return None
-    ptrs = [o.data_ptr() for o in run.outs]
+    import numpy as np
+    ptrs = np.array([o.data_ptr() for o in run.outs], dtype=np.uint64)
     slot = sum(n * run.w.elem_bytes for n in run.numels)
     counter = [100]
 
@@ -968,13 +969,54 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
         for l, n in enumerate(run.numels):
             hviews[l].copy_(device_view(newest[l], n, run.w.dtype).view(tdt))
         torch.cuda.synchronize()
-        cl = run.window if run.window < run.n_feat else chunk_layers
+        # at most 16 chunks: a cache of thousands of small tensors moves in spans, not in
+        # thousands of copies and calls
+        cl = run.window if run.window < run.n_feat else max(chunk_layers, -(-L // 16))
         chunks = [list(range(c, min(c + cl, L))) for c in range(0, L, cl)]
         s_in, s_fc, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         done_out = [None] * len(chunks)
         shared_outs = run.window < run.n_feat
 
         ring_mode = host_bytes < total
+        slot_offs = bc.bc_cache_layout(run.h, L)
+
+        def out_of(l, ls):
+            return run.outs[l - ls[0] if shared_outs else l]
+
+        def spans(ls, dev_addr):
+            """Runs of consecutive layers of `ls` contiguous both in the host buffer and at
+            the device addresses dev_addr(l): (first layer, elements)."""
+            out, l0, n = [], ls[0], run.numels[ls[0]]
+            for l in ls[1:]:
+                if (offs[l] == offs[l - 1] + sizes[l - 1] and
+                        dev_addr(l) == dev_addr(l - 1) + sizes[l - 1]):
+                    n += run.numels[l]
+                else:
+                    out.append((l0, n))
+                    l0, n = l, run.numels[l]
+            out.append((l0, n))
+            return out
+
+        in_spans = [spans(ls, lambda l: slot_offs[l]) for ls in chunks]
+        out_spans = [[(l0, n, out_of(l0, ls).data_ptr()) for l0, n in
+                      spans(ls, lambda l, ls=ls: out_of(l, ls).data_ptr())] for ls in chunks]
+        chunk_ptrs = []
+        for ls in chunks:
+            a = np.zeros(L, dtype=np.uint64)
+            for l in ls:
+                a[l] = out_of(l, ls).data_ptr()
+            chunk_ptrs.append(a)
+
+        def h2d(c, slots):
+            for l0, n in in_spans[c]:
+                device_view(slots[l0], n, run.w.dtype).view(tdt).copy_(
+                    torch.from_numpy(host[offs[l0]:offs[l0] + n * eb]).view(tdt),
+                    non_blocking=True)
+
+        def d2h(c):
+            for l0, n, ptr in out_spans[c]:
+                torch.from_numpy(host[offs[l0]:offs[l0] + n * eb]).view(tdt).copy_(
+                    device_view(ptr, n, run.w.dtype).view(tdt), non_blocking=True)
 
         def one_step_ring(i):
             # Layers share host buffers: upload, forecast and read back one chunk at a time,
@@ -984,16 +1026,10 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
             bc.bc_cache_commit(run.h, t_full)
             with torch.cuda.stream(s_fc):
                 for c, ls in enumerate(chunks):
-                    for l in ls:
-                        device_view(slots[l], run.numels[l], run.w.dtype).view(tdt).copy_(
-                            hviews[l], non_blocking=True)
-                    ptrs = [None] * L
-                    for l in ls:
-                        ptrs[l] = run.outs[l - ls[0] if shared_outs else l].data_ptr()
-                    bc.bc_forecast(run.h, t_target, ptrs, run.out_dtype, s_fc.cuda_stream)
-                    for l in ls:
-                        hviews[l].copy_(run.outs[l - ls[0] if shared_outs else l],
-                                        non_blocking=True)
+                    h2d(c, slots)
+                    bc.bc_forecast(run.h, t_target, chunk_ptrs[c], run.out_dtype,
+                                   s_fc.cuda_stream)
+                    d2h(c)
                 ev = torch.cuda.Event()
                 ev.record(s_fc)
                 done_out[-1] = ev
@@ -1008,9 +1044,7 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
                 with torch.cuda.stream(s_in):
                     if done_out[c] is not None:
                         s_in.wait_event(done_out[c])
-                    for l in ls:
-                        device_view(slots[l], run.numels[l], run.w.dtype).view(tdt).copy_(
-                            hviews[l], non_blocking=True)
+                    h2d(c, slots)
                     ev = torch.cuda.Event()
                     ev.record(s_in)
                     landed.append(ev)
@@ -1021,17 +1055,12 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
                     prev = done_out[c - 1] if c > 0 else done_out[-1]
                     if prev is not None:
                         s_fc.wait_event(prev)
-                ptrs = [None] * L
-                for l in ls:
-                    ptrs[l] = run.outs[l - ls[0] if shared_outs else l].data_ptr()
-                bc.bc_forecast(run.h, t_target, ptrs, run.out_dtype, s_fc.cuda_stream)
+                bc.bc_forecast(run.h, t_target, chunk_ptrs[c], run.out_dtype, s_fc.cuda_stream)
                 ev = torch.cuda.Event()
                 ev.record(s_fc)
                 with torch.cuda.stream(s_out):
                     s_out.wait_event(ev)
-                    for l in ls:
-                        hviews[l].copy_(run.outs[l - ls[0] if shared_outs else l],
-                                        non_blocking=True)
+                    d2h(c)
                     ev2 = torch.cuda.Event()
                     ev2.record(s_out)
                     done_out[c] = ev2

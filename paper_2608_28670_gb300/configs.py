@@ -1,8 +1,9 @@
-"""The five synthetic forecast workloads and their sampling schedules.
+"""The synthetic forecast workloads and their sampling schedules.
 
 Shapes follow the DiT families the paper evaluates (Sec. 4.1): DiT-XL/2 class-to-image,
 PixArt text-to-image, a large MMDiT text-to-image model and HunyuanVideo-class
-text-to-video, each cached as a list of per-block feature tensors.  Values are synthetic
+text-to-video, each cached as a list of per-block feature tensors, plus the many-tensor
+blockwise cache of Sec. 4.5.  Values are synthetic
 (no model weights): per-element random polynomial trajectories in time plus noise
 (:mod:`.synth`).  The schedule is the equal-spaced one of Sec. 3.3: a full step every
 ``interval`` steps, plus the first K steps to fill the window; every other step is a cache
@@ -147,6 +148,10 @@ WORKLOADS: dict[str, Workload] = {
     # 2..4, 50-step flow schedule forecasting 2 of every 3 steps.
     "t2v": Workload("t2v", (1, 118800, 3072), 60, DTYPE_BF16, 3, 50, 3, "flow", 2, 1e-2,
                     K_sweep=(2, 3, 4)),
+    # Blockwise (module-level) cache of Sec. 4.5 / Tables 5-6: many small tensors instead of
+    # one per block -- 4096 tensors of 65,536 bf16 elements, K = 3 (1.6 GB of cache), the
+    # per-tensor forecast of every one in one launch.
+    "blockwise": Workload("blockwise", (65536,), 4096, DTYPE_BF16, 3, 20, 3, "flow", 2, 1e-2),
 }
 
 # Device-memory budget of the video workload (cache + forecast output) stated with it.

@@ -57,8 +57,12 @@ class WorkloadRun:
             self.window = int(window)
             self.calls = -(-self.n_feat // self.window)
             tdt = torch.float32 if self.out_dtype == bc.DTYPE_F32 else torch.bfloat16
-            self.outs = [torch.empty(w.layer_numel, dtype=tdt, device="cuda")
-                         for _ in range(self.window)]
+            # one buffer, each window layer's output at a 256-byte aligned offset, so that
+            # consecutive outputs can also be moved as one span
+            stride = -(-w.layer_numel * out_eb // 256) * 256 // out_eb
+            self._out_flat = torch.empty(stride * self.window, dtype=tdt, device="cuda")
+            self.outs = [self._out_flat[i * stride:i * stride + w.layer_numel]
+                         for i in range(self.window)]
             # per-call output tables, built once (the binding passes numpy tables as is)
             self._call_ptrs = [np.array([q or 0 for q in self.out_ptrs(c)], dtype=np.uint64)
                                for c in range(self.calls)]
@@ -138,4 +142,5 @@ class WorkloadRun:
             bc.bc_cache_destroy(self.h)
             self.h = 0
         self.outs = []
+        self._out_flat = None
         self.x = None

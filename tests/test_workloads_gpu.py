@@ -103,8 +103,9 @@ def test_c2i_256_every_element():
         run.close()
 
 
-@pytest.mark.parametrize("name", ["c2i-512", "t2i-1024", "mmdit-t2i"])
+@pytest.mark.parametrize("name", ["c2i-512", "t2i-1024", "mmdit-t2i", "blockwise"])
 def test_image_workloads_every_element(name):
+    # (blockwise: 4096 tensors, one launch through the device layer table)
     torch.cuda.empty_cache()
     run = WorkloadRun(WORKLOADS[name], stream=stream())
     try:
@@ -112,6 +113,7 @@ def test_image_workloads_every_element(name):
         check_run(run, np.random.default_rng(len(name)))
         st = run.stats()
         assert st["kernel_launches"] == 1 and st["forecasts"] == 1
+        assert st["table_uploads"] == (1 if run.n_feat > 1016 else 0)
     finally:
         run.close()
         torch.cuda.empty_cache()
