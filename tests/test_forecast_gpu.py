@@ -363,6 +363,73 @@ def test_many_layers_in_a_graph_carry_their_own_tables(kernel):
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+def test_many_layers_with_the_sampler_update(kernel):
+    # 1200 layers, the model output among them (index 1100): the fused a x + b v_hat + c z
+    # update rides in the one device-table launch; under graph capture the launch is split
+    # and the update layer lands in the second parameter-block group.  Both must match the
+    # oracle, and the replay the eager result bit for bit.
+    numels = [(i * 29) % 513 + 16 for i in range(1200)]
+    numels[1100] = 40_000 + 3
+    K, times, t_new = 3, [0.9, 0.85, 0.8], 0.75
+    feats = synth.host_trajectories([(n,) for n in numels], times, dtype="bf16", seed=41)
+    h = bc.bc_cache_create(numels, K, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
+    try:
+        for t, per in zip(times, feats):
+            dev = [to_device(f) for f in per]
+            bc.bc_cache_push(h, [d.data_ptr() for d in dev], t, stream())
+            torch.cuda.synchronize()
+        a, b, c = 0.98, -0.05, 0.02
+        x0 = np.linspace(-1.0, 1.0, numels[1100]).astype(np.float32)
+        z = np.cos(np.arange(numels[1100])).astype(np.float32)
+        zd = to_device(z)
+        outs = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        for o in outs:
+            o.fill_(0)                  # outs[1100] is never written (the update layer)
+        ptrs = [o.data_ptr() for o in outs]
+        ptrs[1100] = None
+        x = to_device(x0)
+        l0 = bc.bc_cache_stats(h)["kernel_launches"]
+        bc.bc_forecast_update(h, t_new, a, b, c, ptrs, bc.DTYPE_BF16, 1100, x.data_ptr(),
+                              bc.DTYPE_F32, zd.data_ptr(), stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["kernel_launches"] - l0 == 1
+        W = oracle.paper_weights(times[::-1], t_new)
+        nf = feats[::-1]
+        x_ref, xb = oracle.update([f[1100] for f in nf], W, x0, a, b, c, z)
+        assert_close(to_host(x, bc.DTYPE_F32), x_ref, xb, bc.DTYPE_F32, "x")
+        for l in (0, 1099, 1101, 1199):
+            ref, bound = oracle.combine([f[l] for f in nf], W)
+            assert_close(to_host(outs[l], bc.DTYPE_BF16), ref, bound, bc.DTYPE_BF16, f"layer {l}")
+        eager_x = x.clone()
+        eager_outs = [o.clone() for o in outs]
+        # the same call captured into a graph (parameter-block launches of <= 1016 layers)
+        for sel in (1000, 190):                 # first uses of those launchers, uncaptured
+            bc.bc_forecast(h, t_new, [q if i < sel else None for i, q in enumerate(ptrs)],
+                           bc.DTYPE_BF16, stream())
+        x.copy_(to_device(x0))
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        s_ = torch.cuda.Stream()
+        with torch.cuda.stream(s_):
+            with torch.cuda.graph(g, stream=s_, capture_error_mode="thread_local"):
+                bc.bc_forecast_update(h, t_new, a, b, c, ptrs, bc.DTYPE_BF16, 1100, x.data_ptr(),
+                                      bc.DTYPE_F32, zd.data_ptr(), s_.cuda_stream)
+        for o in outs:
+            o.fill_(0)
+        x.copy_(to_device(x0))
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(x, eager_x)
+        for p_, q_ in zip(outs, eager_outs):
+            assert torch.equal(p_, q_)
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
 @pytest.mark.parametrize("in_dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
 @pytest.mark.parametrize("K", [1, 2, 3, 4])
 def test_small_launch_half_tiles_match_the_register_kernel(in_dt, K):
