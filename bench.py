@@ -921,6 +921,41 @@ def pinned_host_buffer(nbytes):
     return arr, (lambda: cudart.cudaHostUnregister(arr.ctypes.data)), "cudaHostRegister"
 
 
+def link_probe(host, nbytes, probe_bytes=4 * 10**9):
+    """Copy-engine throughput of this machine's host link on the e2e leg's own pinned buffer: H2D,
+    D2H, and both at once (two streams, half the bytes each way), GB/s."""
+    import torch
+    n = min(int(nbytes), int(probe_bytes)) // 4096 * 4096
+    if n < 2 * 4096:
+        return None
+    hv = torch.from_numpy(host[:n])
+    dev = torch.empty(n, dtype=torch.uint8, device="cuda")
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        fn()
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0
+
+    half = n // 2
+
+    def both():
+        with torch.cuda.stream(s1):
+            dev[:half].copy_(hv[:half], non_blocking=True)
+        with torch.cuda.stream(s2):
+            hv[half:].copy_(dev[half:], non_blocking=True)
+
+    out = {"bytes": n,
+           "h2d_GB/s": round(n / timed(lambda: dev.copy_(hv, non_blocking=True)) / 1e9, 1),
+           "d2h_GB/s": round(n / timed(lambda: hv.copy_(dev, non_blocking=True)) / 1e9, 1),
+           "both_GB/s": round(n / timed(both) / 1e9, 1)}
+    del dev
+    return out
+
+
 def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
     """Same metric through the public API with host buffers.  Per step: the new full-step
     features (one slot, every layer) are copied from pinned host memory into the next cache
@@ -1067,25 +1102,38 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
 
         one_step(0)                      # warm-up
         torch.cuda.synchronize()
+        link = link_probe(host, host_bytes)
         if dist is not None:
             dist.barrier()
         t0 = time.perf_counter()
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
+        marks = []
         a.record()
         for i in range(steps):
             one_step(i + 1)
+            ev = torch.cuda.Event(enable_timing=True)      # this step's last read-back
+            ev.record(s_fc if ring_mode else s_out)
+            marks.append(ev)
         for ev in done_out:
             if ev is not None:
                 torch.cuda.current_stream().wait_event(ev)
         b.record()
         torch.cuda.synchronize()
+        step_marks = [round(a.elapsed_time(m), 1) for m in marks]
         wall = time.perf_counter() - t0
         ms = max_over_ranks(a.elapsed_time(b) / steps, dist)
         alg = run.algorithmic_bytes()
+        moved = total + run.n_feat * run.w.layer_numel * ob
+        link_gbs = moved / (ms * 1e-3) / 1e9
         return {"value": round(job_throughput(alg, ms, world), 1), "unit": "GB/s",
                 "h2d_bytes_per_step": total,
                 "d2h_bytes_per_step": run.n_feat * run.w.layer_numel * ob,
+                "host_link_GB/s": round(link_gbs, 1),
+                "step_end_ms": step_marks,
+                "link_probe": link,
+                "frac_of_link_both": (round(link_gbs / link["both_GB/s"], 3)
+                                      if link and link.get("both_GB/s") else None),
                 "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
                 "chunk_layers": cl, "host_memory": kind, "host_buffer_bytes": int(host_bytes),
                 "overlapped": not ring_mode,
