@@ -191,7 +191,7 @@ bc_status bc_cache_reset(bc_handle h);
  * push has at least 16 tiles of 32 KiB per SM, else register loads and stores.  Beyond 1016
  * layers the launch reads its layer table from the handle's device copy, re-uploaded only
  * when the sources differ from the previous push (outside stream capture; while `stream` is
- * captured, one launch per 1016 layers).  The node
+ * captured, one launch per 1016 layers; ordered across streams as for bc_forecast).  The node
  * counts as pushed when the call returns; if the pipeline copy gives up waiting (reported
  * by bc_cache_check) the slot's contents are undefined and the cache should be reset.  `t`
  * is the timestep of this full step.  Errors: INVALID_ARG (null pointer, non-finite t,
@@ -233,9 +233,12 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  * layers the launch reads its layer table from the handle's device copy, which is
  * re-uploaded (one cudaMemcpyAsync on `stream`, from pinned memory) only when the outputs
  * differ from the previous such call; the host waits only if four uploads of different
- * tables are still queued ahead of the device.  While `stream` is being captured into a CUDA
- * graph it issues one launch per 1016 layers instead, so that the graph holds its own
- * tables.
+ * tables are still queued ahead of the device.  Such a call on another stream than the
+ * previous one first makes `stream` wait (cudaStreamWaitEvent) for the previous launch that
+ * read the table, so forecasts of one handle on several streams never see each other's
+ * tables (their outputs remain the caller's to keep apart).  While `stream` is being
+ * captured into a CUDA graph it issues one launch per 1016 layers instead, so that the
+ * graph holds its own tables.
  * Layers with a NULL output are skipped, which also serves to forecast a window of layers.
  * Outputs must not overlap the arena (checked) or each other (not checked: overlapping
  * outputs race).

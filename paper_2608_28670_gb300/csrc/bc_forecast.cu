@@ -205,6 +205,14 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
          count_tiles(layers, n, T::kBytes, kCopyTileBytes / kVecBytes) >=
              static_cast<int64_t>(kCopyMinTilesPerCta) * sms);
     const int tile_groups = pipeline ? kCopyTileBytes / 16 : kThreads * kCopyVecsPerThread;
+    // the launch's error, after recording that a device-table launch reads its table
+    auto launched = [&](cudaError_t e) -> int {
+        if constexpr (CAP == 0) {
+            const int r = table_used(*opt.table, s);
+            if (e == cudaSuccess) return r;
+        }
+        return e;
+    };
     if constexpr (CAP == 0) {
         std::vector<LayerEntry> &tab = table_scratch();
         tab.resize(static_cast<size_t>(n));
@@ -231,14 +239,14 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
         kern<<<grid, kCopyTmaThreads, kCopySmemBytes, s>>>(a);
         ++*launches;
         ++*pipeline_launches;
-        return cudaGetLastError();
+        return launched(cudaGetLastError());
     }
     auto kern = copy_kernel<T, CAP>;
     const int64_t cap = static_cast<int64_t>(sms) * resident_ctas(kern, occ, 0);
     const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
     kern<<<grid, kThreads, 0, s>>>(a);
     ++*launches;
-    return cudaGetLastError();
+    return launched(cudaGetLastError());
 }
 
 template <class T>

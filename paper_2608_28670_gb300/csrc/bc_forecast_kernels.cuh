@@ -714,11 +714,18 @@ inline int64_t fill_entries(LayerEntry *dst, const LayerEntry *layers, int n, in
     return tiles;
 }
 
-// Make the handle's device table hold `entries[0..n)`: one cudaMemcpyAsync on `s` from the
-// next pinned staging buffer, skipped when the previous upload was the same table.  A staging
-// buffer is rewritten only after the copy that last read it has run (its event).
+// Make the handle's device table hold `entries[0..n)` for a launch on `s`: one
+// cudaMemcpyAsync on `s` from the next pinned staging buffer, skipped when the previous upload
+// was the same table.  A staging buffer is rewritten only after the copy that last read it has
+// run (its event).  When the last launch that read the table went to another stream, `s`
+// first waits for it: that launch may still be reading the table this copy overwrites, and
+// a launch that reuses the table must follow the copy queued on that stream ahead of it.
 inline int upload_table(DeviceTable &tb, const LayerEntry *entries, int n, cudaStream_t s) {
     const size_t bytes = sizeof(LayerEntry) * static_cast<size_t>(n);
+    if (tb.used_recorded && tb.used_stream != static_cast<void *>(s)) {
+        const cudaError_t e = cudaStreamWaitEvent(s, static_cast<cudaEvent_t>(tb.used), 0);
+        if (e != cudaSuccess) return e;
+    }
     if (tb.valid == n && tb.last >= 0 &&
         std::memcmp(tb.host + static_cast<size_t>(tb.last) * tb.capacity, entries, bytes) == 0)
         return cudaSuccess;
@@ -740,6 +747,15 @@ inline int upload_table(DeviceTable &tb, const LayerEntry *entries, int n, cudaS
     tb.last = k;
     tb.valid = n;
     ++tb.uploads;
+    return cudaSuccess;
+}
+
+// Record that a launch on `s` reads the table (after the launch, on `s`).
+inline int table_used(DeviceTable &tb, cudaStream_t s) {
+    const cudaError_t e = cudaEventRecord(static_cast<cudaEvent_t>(tb.used), s);
+    if (e != cudaSuccess) return e;
+    tb.used_stream = s;
+    tb.used_recorded = true;
     return cudaSuccess;
 }
 
@@ -806,6 +822,14 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
             static_cast<int64_t>(BC_SMALL_LAUNCH_TILES_PER_SM) * sms)
         vpt = 1;
     const int tile_vecs = kThreads * (pipeline ? kTmaVpt<K> : vpt);
+    // the launch's error, after recording that a device-table launch reads its table
+    auto launched = [&](cudaError_t e) -> int {
+        if constexpr (CAP == 0) {
+            const int r = table_used(*p.table, s);
+            if (e == cudaSuccess) return r;
+        }
+        return e;
+    };
 
     if constexpr (CAP == 0) {
         std::vector<LayerEntry> &tab = table_scratch();
@@ -840,7 +864,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
         kern<<<grid, kThreads, smem, s>>>(a);
         ++*launches;
         ++*pipeline_launches;
-        return cudaGetLastError();
+        return launched(cudaGetLastError());
     }
     if constexpr (CAP == kLayersSmall && kRegVpt > 1) {
         if (vpt == 1) {
@@ -860,7 +884,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
     const int grid = static_cast<int>(a.total_tiles < cap ? a.total_tiles : cap);
     kern<<<grid, kThreads, 0, s>>>(a);
     ++*launches;
-    return cudaGetLastError();
+    return launched(cudaGetLastError());
 }
 
 template <int K, class TIn, class TOut>

@@ -257,10 +257,13 @@ bc_status alloc_table(bc::DeviceTable &tb, int n_layers) {
     if (e == cudaSuccess) e = cudaHostAlloc(&host, bytes * bc::kTableStaging, cudaHostAllocDefault);
     for (int k = 0; k < bc::kTableStaging && e == cudaSuccess; ++k)
         e = cudaEventCreateWithFlags(&ev[k], cudaEventDisableTiming);
+    cudaEvent_t used = nullptr;
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&used, cudaEventDisableTiming);
     if (e != cudaSuccess) {
         cudaGetLastError();
         for (int k = 0; k < bc::kTableStaging; ++k)
             if (ev[k]) cudaEventDestroy(ev[k]);
+        if (used) cudaEventDestroy(used);
         if (dev) cudaFree(dev);
         if (host) cudaFreeHost(host);
         return e == cudaErrorMemoryAllocation ? fail(BC_ERR_OOM, "layer table")
@@ -269,6 +272,7 @@ bc_status alloc_table(bc::DeviceTable &tb, int n_layers) {
     tb.dev = static_cast<bc::LayerEntry *>(dev);
     tb.host = static_cast<bc::LayerEntry *>(host);
     for (int k = 0; k < bc::kTableStaging; ++k) tb.uploaded[k] = ev[k];
+    tb.used = used;
     tb.capacity = n_layers;
     return BC_OK;
 }
@@ -288,6 +292,7 @@ cudaError_t free_table(bc::DeviceTable &tb) {
     if (tb.host) keep(cudaFreeHost(tb.host));
     for (int k = 0; k < bc::kTableStaging; ++k)
         if (tb.uploaded[k]) keep(cudaEventDestroy(static_cast<cudaEvent_t>(tb.uploaded[k])));
+    if (tb.used) keep(cudaEventDestroy(static_cast<cudaEvent_t>(tb.used)));
     tb = bc::DeviceTable{};
     return rc;
 }

@@ -104,7 +104,9 @@ static_assert(sizeof(ForecastArgs<kLayersLarge>) <= 32764, "layer table exceeds 
 // differs from the previous upload: a sampler that reuses its buffers uploads once.  The
 // pinned staging is a ring of kTableStaging buffers, each reused only after the copy that
 // last read it has run (its event), so the host waits only if that many uploads with
-// different tables are still queued ahead of the device.
+// different tables are still queued ahead of the device.  An event recorded after every
+// launch that reads the table lets a call on another stream wait (on the device) until that
+// launch is done, before it rewrites the table or reads the copy queued ahead of it.
 constexpr int kTableStaging = 4;
 struct DeviceTable {
     LayerEntry *dev = nullptr;     // device, `capacity` entries
@@ -114,6 +116,9 @@ struct DeviceTable {
     int last = -1;                 // staging buffer of the last upload
     bool pending[kTableStaging] = {};        // an event was recorded after the buffer's copy
     void *uploaded[kTableStaging] = {};      // cudaEvent_t per staging buffer
+    void *used = nullptr;          // cudaEvent_t recorded after the last launch that read `dev`
+    void *used_stream = nullptr;   // that launch's stream
+    bool used_recorded = false;
     int64_t uploads = 0;           // uploads so far
 };
 

@@ -364,6 +364,55 @@ def test_many_layers_in_a_graph_carry_their_own_tables(kernel):
 
 
 @pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+def test_many_layers_on_two_streams_share_the_device_table(kernel):
+    # Forecasts over more layers than a parameter block holds read the handle's one device
+    # table.  Issued on two streams without the caller's synchronisation, a call on the other
+    # stream must wait for the last launch that read the table: before rewriting it (new
+    # outputs) and before reusing the copy queued on that stream.  2048 layers of 32 Ki bf16
+    # (512 MiB moved per forecast) keep each launch long enough for a missing wait to show.
+    n_l, n = 2048, 32768
+    K = 3
+    h = bc.bc_cache_create([n] * n_l, K, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
+    s0 = stream()
+    try:
+        for j, tau in enumerate((0.9, 0.85, 0.8)):
+            slots = bc.bc_cache_next_slot_ptrs(h, n_l)
+            offs = bc.bc_cache_layout(h, n_l)
+            synth.fill_device(slots[0], bc.DTYPE_BF16, offs[-1] // 2, seed=21, tensor_id=0,
+                              step_id=j, tau=tau, degree=2, noise_std=1e-2, stream=s0)
+            bc.bc_cache_commit(h, tau)
+        t1, t2 = 0.75, 0.7
+        ref = {t: [torch.empty(n, dtype=torch.bfloat16, device="cuda") for _ in range(n_l)]
+               for t in (t1, t2)}
+        for t, outs in ref.items():
+            bc.bc_forecast(h, t, [o.data_ptr() for o in outs], bc.DTYPE_BF16, s0)
+        torch.cuda.synchronize()
+        assert not torch.equal(ref[t1][0], ref[t2][0])
+        o1, o2, o3 = ([torch.full((n,), 3.0, dtype=torch.bfloat16, device="cuda")
+                       for _ in range(n_l)] for _ in range(3))
+        torch.cuda.synchronize()
+        sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+        ptr = lambda outs: [o.data_ptr() for o in outs]          # noqa: E731
+        st0 = bc.bc_cache_stats(h)
+        bc.bc_forecast(h, t1, ptr(o1), bc.DTYPE_BF16, sa.cuda_stream)   # upload on a
+        bc.bc_forecast(h, t2, ptr(o2), bc.DTYPE_BF16, sb.cuda_stream)   # rewrite on b
+        bc.bc_forecast(h, t2, ptr(o3), bc.DTYPE_BF16, sa.cuda_stream)   # rewrite on a
+        bc.bc_forecast(h, t1, ptr(o3), bc.DTYPE_BF16, sb.cuda_stream)   # reuse on b, after a
+        torch.cuda.synchronize()
+        st1 = bc.bc_cache_stats(h)
+        assert st1["table_uploads"] - st0["table_uploads"] == 3
+        assert st1["kernel_launches"] - st0["kernel_launches"] == 4
+        for got, want in ((o1, ref[t1]), (o2, ref[t2]), (o3, ref[t1])):
+            for l in range(n_l):
+                assert torch.equal(got[l], want[l]), f"layer {l}"
+        bc.bc_cache_check(h)
+    finally:
+        torch.cuda.synchronize()
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 def test_many_layers_with_the_sampler_update(kernel):
     # 1200 layers, the model output among them (index 1100): the fused a x + b v_hat + c z
     # update rides in the one device-table launch; under graph capture the launch is split
