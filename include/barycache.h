@@ -30,14 +30,16 @@
  *  - CUDA graphs: while `stream` is being captured, pushes, commits, forecasts (all
  *    variants) and the probe drift enqueue kernels only (no allocation, copy or
  *    synchronisation), so they may be called during capture (outside capture, a forecast or
- *    push over more than 1016 layers may also copy its layer table to the device).  The graph holds the slot addresses, weights and update
- *    coefficients chosen when each call was made; replaying it repeats that device work
- *    and does not move the handle's host state (ring head, node times, statistics).  The
- *    first forecast of each kind on a device also queries and sets per-device kernel
- *    attributes; run the loop once uncaptured before capturing it.
+ *    push over more than 1016 layers may also copy its layer table to the device).  The
+ *    graph holds the slot addresses, weights and update coefficients chosen when each call
+ *    was made; replaying it repeats that device work and does not move the handle's host
+ *    state (ring head, node times, statistics).  The first forecast of each kind on a
+ *    device also queries and sets per-device kernel attributes; run the loop once
+ *    uncaptured before capturing it.
  *  - Host-side cache state (ring head, node times) changes when the call is made, so
  *    pushes and forecasts on one handle must be issued from one thread, in order, on one
- *    stream (or with the caller's own synchronisation).
+ *    stream (or with the caller's own synchronisation between a push and the calls that
+ *    read its slot).  The library orders only its own layer tables across streams.
  *  - No exception crosses the ABI and device code never traps.  The pipeline forecast
  *    kernel and the large drift and push kernels wait on their own shared-memory
  *    pipelines (TMA bulk copies completing on mbarriers); every such wait gives up after
@@ -331,11 +333,11 @@ bc_status bc_adaptive_decide(bc_adaptive *s, double drift, int *run_full);
 
 /* The probe drift of the adaptive schedule, on the device:
  *     out[0] = sum_e |cur[e] - prev[e]|,  out[1] = sum_e |prev[e]|,  out[2] = out[0]/out[1]
- * (out[2] = 0 when both sums are 0, +inf when only out[1] is, NaN when either sum is NaN).  cur, prev: device, n
- * elements of dtype, 16-byte aligned; out: 3 device doubles.  Two launches on `stream` with
- * a fixed reduction order (bitwise reproducible on one device for a given kernel choice),
- * using the handle's reduction scratch, so calls on one handle must not overlap on the
- * device.  If the pipeline form gives up waiting (see bc_cache_check), out[] reads NaN.  The
+ * (out[2] = 0 when both sums are 0, +inf when only out[1] is, NaN when either sum is NaN).
+ * cur, prev: device, n elements of dtype, 16-byte aligned; out: 3 device doubles.  Two
+ * launches on `stream` with a fixed reduction order (bitwise reproducible on one device for
+ * a given kernel choice), using the handle's reduction scratch, so calls on one handle must
+ * not overlap on the device.  If the pipeline form gives up waiting (see bc_cache_check), out[] reads NaN.  The
  * caller reads out[2] back to drive bc_adaptive_decide.  Errors: INVALID_ARG, ALIGNMENT,
  * CUDA. */
 bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
