@@ -413,6 +413,43 @@ def test_many_layers_on_two_streams_share_the_device_table(kernel):
 
 
 @pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+def test_many_layer_pushes_on_two_streams_share_the_push_table(kernel):
+    # The push table of a cache over 1016 layers, used from two streams: each push on the
+    # other stream must wait for the last copy that read the table (new sources rewrite it;
+    # reused sources must follow the upload queued on the other stream).  Every slot must
+    # hold exactly the bytes of the sources pushed into it.
+    n_l, n = 2048, 32768
+    h = bc.bc_cache_create([n] * n_l, 3, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
+    try:
+        rng = np.random.default_rng(29)
+        srcs = [to_device(rng.integers(0, 2 ** 16, n * n_l, dtype=np.uint16)) for _ in range(3)]
+        ptrs = [np.array([s_.data_ptr() + 2 * n * l for l in range(n_l)], dtype=np.uint64)
+                for s_ in srcs]
+        torch.cuda.synchronize()
+        sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+        st0 = bc.bc_cache_stats(h)
+        bc.bc_cache_push(h, ptrs[0], 0.9, sa.cuda_stream)     # upload on a
+        bc.bc_cache_push(h, ptrs[1], 0.8, sb.cuda_stream)     # rewrite on b
+        bc.bc_cache_push(h, ptrs[2], 0.7, sa.cuda_stream)     # rewrite on a
+        bc.bc_cache_push(h, ptrs[2], 0.6, sb.cuda_stream)     # reuse on b, after a
+        torch.cuda.synchronize()
+        bc.bc_cache_check(h)
+        st1 = bc.bc_cache_stats(h)
+        assert st1["table_uploads"] - st0["table_uploads"] == 3
+        assert st1["kernel_launches"] - st0["kernel_launches"] == 4
+        assert bc.bc_cache_nodes(h) == [0.6, 0.7, 0.8]
+        for j, want in enumerate((srcs[2], srcs[2], srcs[1])):
+            slots = bc.bc_cache_slot_ptrs(h, j, n_l)
+            for l in range(n_l):
+                got = device_view(slots[l], n, bc.DTYPE_BF16)
+                assert torch.equal(got, want[l * n:(l + 1) * n]), f"node {j} layer {l}"
+    finally:
+        torch.cuda.synchronize()
+        bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 def test_many_layers_with_the_sampler_update(kernel):
     # 1200 layers, the model output among them (index 1100): the fused a x + b v_hat + c z
     # update rides in the one device-table launch; under graph capture the launch is split
