@@ -717,7 +717,8 @@ def time_blockwise(stream, steps):
     """Row f2: a many-tensor (blockwise) cache -- 4096 tensors of 65,536 bf16 elements, K = 3
     (1.6 GB of cache) -- forecast through per-layer output pointers (one launch reading its
     layer table from the handle's device copy, uploaded once for these outputs) and through
-    one flat slot-shaped output (one launch)."""
+    one flat slot-shaped output (one launch); its full-step push from per-tensor sources and
+    from one slot-shaped buffer (bc_cache_push_flat)."""
     import numpy as np
     import torch
     from paper_2608_28670_gb300 import barycache as bc
@@ -776,6 +777,13 @@ def time_blockwise(stream, steps):
         bc.bc_cache_set_kernel(h, bc.KERNEL_AUTO)
         ms_push = timed(push)
         push_launches = timed.launches
+        uploads = bc.bc_cache_stats(h)["table_uploads"] - st["table_uploads"]
+
+        def push_flat():            # the same step from one slot-shaped buffer
+            bc.bc_cache_push_flat(h, flat.data_ptr(), push_t[k[0]], stream)
+            k[0] += 1
+        ms_push_flat = timed(push_flat)
+        push_flat_launches = timed.launches
         return {"tensors": n_t, "elements_per_tensor": n,
                 "per_layer": {"GB/s": round(alg / (ms_layers * 1e-3) / 1e9, 1),
                               "ms": round(ms_layers, 4),
@@ -788,8 +796,10 @@ def time_blockwise(stream, steps):
                          "ms": round(ms_push, 4), "launches_per_call": push_launches,
                          "GB/s_by_kernel": push_by_kernel,
                          "bytes_per_push": push_bytes,
-                         "table_uploads": bc.bc_cache_stats(h)["table_uploads"]
-                                          - st["table_uploads"]}}
+                         "table_uploads": uploads},
+                "push_flat": {"GB/s": round(push_bytes / (ms_push_flat * 1e-3) / 1e9, 1),
+                              "ms": round(ms_push_flat, 4),
+                              "launches_per_call": push_flat_launches}}
     finally:
         bc.bc_cache_destroy(h)
 

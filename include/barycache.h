@@ -282,6 +282,15 @@ bc_status bc_forecast_update(bc_handle h, double t_new, double a, double b, doub
  * written with unspecified values.  Errors as bc_forecast. */
 bc_status bc_forecast_flat(bc_handle h, double t_new, void *out, void *stream);
 
+/* Full-step push (Eq. 6) from one device buffer laid out like a cache slot (layer l at byte
+ * offset offsets[l] of bc_cache_layout, in the cache dtype, offsets[n_layers] bytes in all,
+ * 16-byte aligned): the oldest slot is evicted and the whole buffer, padding included, is
+ * copied into it by one byte-exact copy launch, whatever the number of layers, with no
+ * per-layer table (the push counterpart of bc_forecast_flat).  Kernel choice, stream
+ * semantics and the give-up behaviour as bc_cache_push.  Errors: INVALID_ARG (NULL src,
+ * non-finite t, src overlapping the arena), ALIGNMENT, DUPLICATE_NODE, CUDA. */
+bc_status bc_cache_push_flat(bc_handle h, const void *src, double t, void *stream);
+
 /* Byte offset of every layer inside a slot (and inside a bc_forecast_flat output), in
  * offsets[0 .. n_layers-1]; offsets[n_layers] = bytes per slot. */
 bc_status bc_cache_layout(bc_handle h, int64_t *offsets);
@@ -375,7 +384,8 @@ bc_status bc_cache_check(bc_handle h);
  * every CTA's pipeline unarmed, so that its bounded wait runs out (about one second) and the
  * launch returns early with the status word set, which bc_cache_check then reports;
  * what = 2 does the same to the next probe drift of at least one 16 KiB tile (its out[]
- * then reads NaN); what = 3 to the next push copy (the pushed slot is then undefined);
+ * then reads NaN); what = 3 to the next push copy (bc_cache_push or bc_cache_push_flat;
+ * the pushed slot is then undefined);
  * what = 0 cancels a pending injection.  Nothing is faulted: the copies
  * that were issued complete and are drained. */
 bc_status bc_cache_inject_fault(bc_handle h, int what);

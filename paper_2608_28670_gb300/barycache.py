@@ -92,6 +92,8 @@ _SIGNATURES = {
                             ctypes.c_double, ctypes.POINTER(ctypes.c_void_p), ctypes.c_int,
                             ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
                             ctypes.c_void_p], ctypes.c_int),
+    "bc_cache_push_flat": ([ctypes.c_void_p, ctypes.c_void_p, ctypes.c_double, ctypes.c_void_p],
+                           ctypes.c_int),
     "bc_forecast_flat": ([ctypes.c_void_p, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p],
                          ctypes.c_int),
     "bc_cache_layout": ([ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)], ctypes.c_int),
@@ -264,6 +266,11 @@ def bc_cache_info(h: int) -> tuple[int, int, int]:
 def bc_cache_push(h: int, layer_ptrs: Sequence[int], t: float, stream: int = 0) -> None:
     _check(lib().bc_cache_push(h, _layer_ptrs(h, layer_ptrs, "bc_cache_push"), float(t),
                                stream or None), "bc_cache_push")
+
+
+def bc_cache_push_flat(h: int, src: int, t: float, stream: int = 0) -> None:
+    _check(lib().bc_cache_push_flat(h, src or None, float(t), stream or None),
+           "bc_cache_push_flat")
 
 
 def bc_cache_next_slot_ptrs(h: int, n_layers: int | None = None) -> list[int]:

@@ -728,6 +728,40 @@ bc_status bc_cache_push(bc_handle h, const void *const *layer_ptrs, double t, vo
     }
 }
 
+bc_status bc_cache_push_flat(bc_handle h, const void *src, double t, void *stream) {
+    t_last_error.clear();
+    try {
+        bc_status s = check_handle(h);
+        if (s != BC_OK) return s;
+        if (!src) return fail(BC_ERR_INVALID_ARG, "src is NULL");
+        if (!aligned16(src)) return fail(BC_ERR_ALIGNMENT, "src is not 16-byte aligned");
+        if (h->overlaps_arena(reinterpret_cast<uint64_t>(src), h->slot_bytes))
+            return fail(BC_ERR_INVALID_ARG, "src overlaps the cache arena");
+        s = check_new_node(h, t);
+        if (s != BC_OK) return s;
+        if (h->slot_bytes > 0) {
+            const int next = (h->head + 1) % h->K;
+            bc::LayerEntry e{};
+            e.src = reinterpret_cast<uint64_t>(src);
+            e.dst = 0;
+            e.numel = static_cast<int64_t>(h->slot_bytes / elem_bytes(h->dtype));
+            DeviceGuard g(h->device);
+            if (!g.ok) return fail(BC_ERR_CUDA, "cannot select the cache's device");
+            bc::CopyOptions opt{h->kernel, h->status, h->inject_next_push ? 1 : 0, nullptr,
+                                reinterpret_cast<uint64_t>(h->slot_base(next))};
+            const int err = bc::launch_copy(&e, 1, h->dtype, opt, stream,
+                                            &h->stats.kernel_launches,
+                                            &h->stats.pipeline_launches);
+            h->inject_next_push = false;
+            if (err != cudaSuccess) return cuda_fail(err, "push copy launch");
+        }
+        rotate_in(h, t);
+        return BC_OK;
+    } catch (...) {
+        return fail(BC_ERR_INVALID_ARG, "internal exception");
+    }
+}
+
 bc_status bc_cache_next_slot_ptrs(bc_handle h, void **out_ptrs) {
     t_last_error.clear();
     bc_status s = check_handle(h);

@@ -83,6 +83,17 @@ def test_pointer_checks():
         assert _status(bc.bc_forecast, h, float("inf"), [p, None], bc.DTYPE_BF16, s()) == \
             bc.ERR_INVALID_ARG
         assert _status(bc.bc_cache_slot_ptrs, h, 1, 2) == bc.ERR_INVALID_ARG
+        # the flat push: one slot image of 8192 + 256 bytes
+        assert bc.bc_cache_layout(h)[-1] <= x.numel() * 2
+        assert _status(bc.bc_cache_push_flat, h, p + 2, 0.3, s()) == bc.ERR_ALIGNMENT
+        assert _status(bc.bc_cache_push_flat, h, 0, 0.3, s()) == bc.ERR_INVALID_ARG
+        nxt = bc.bc_cache_next_slot_ptrs(h, 2)
+        assert _status(bc.bc_cache_push_flat, h, nxt[0], 0.3, s()) == bc.ERR_INVALID_ARG
+        assert _status(bc.bc_cache_push_flat, h, p, 0.5, s()) == bc.ERR_DUPLICATE_NODE
+        assert _status(bc.bc_cache_push_flat, h, p, float("nan"), s()) == bc.ERR_INVALID_ARG
+        assert bc.bc_cache_nodes(h) == [0.5]                     # nothing was pushed
+        bc.bc_cache_push_flat(h, p, 0.3, s())
+        assert bc.bc_cache_nodes(h) == [0.3, 0.5]
     finally:
         bc.bc_cache_destroy(h)
     torch.cuda.synchronize()                     # the context is still usable
@@ -203,26 +214,35 @@ def test_drift_pipeline_wait_timeout_is_reported_and_recovers():
         bc.bc_cache_destroy(h)
 
 
-def test_push_pipeline_wait_timeout_is_reported_and_recovers():
+@pytest.mark.parametrize("flat", [False, True], ids=["per_layer", "flat"])
+def test_push_pipeline_wait_timeout_is_reported_and_recovers(flat):
     """The push copy's pipeline form under the same test hook: the launch gives up, the
     check reports it once, and the next push on the handle copies every byte."""
     import time
     n = 16384 * 40 + 7
-    src = torch.arange(n, dtype=torch.float32, device="cuda")
+    src = torch.arange(n + 57, dtype=torch.float32, device="cuda")   # a whole 256-byte slot
+
+    def push(t):
+        if flat:
+            bc.bc_cache_push_flat(h, src.data_ptr(), t, s())
+        else:
+            bc.bc_cache_push(h, [src.data_ptr()], t, s())
+
     h = bc.bc_cache_create([n], 2, bc.DTYPE_F32)
     bc.bc_cache_set_kernel(h, bc.KERNEL_PIPELINE)
     try:
+        assert bc.bc_cache_layout(h)[-1] == src.numel() * 4
         bc.bc_cache_inject_fault(h, 3)
         t0 = time.perf_counter()
-        bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())
+        push(0.9)
         assert _status(bc.bc_cache_check, h) == bc.ERR_DEVICE_TIMEOUT
         assert 0.5 < time.perf_counter() - t0 < 1.9
         bc.bc_cache_check(h)
         bc.bc_cache_reset(h)
-        bc.bc_cache_push(h, [src.data_ptr()], 0.9, s())
+        push(0.9)
         bc.bc_cache_check(h)
         got = device_view(bc.bc_cache_slot_ptrs(h, 0, 1)[0], n, bc.DTYPE_F32)
-        assert torch.equal(got, src)
+        assert torch.equal(got, src[:n])
         assert bc.bc_cache_stats(h)["pipeline_launches"] == 2
     finally:
         bc.bc_cache_destroy(h)

@@ -219,6 +219,68 @@ def test_push_copy_is_byte_exact(kernel, dt):
         bc.bc_cache_destroy(h)
 
 
+@pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
+@pytest.mark.parametrize("dt", [bc.DTYPE_BF16, bc.DTYPE_F32])
+def test_flat_push_copies_the_slot_image_byte_exact(kernel, dt):
+    # bc_cache_push_flat copies a slot-shaped buffer (bc_cache_layout offsets, padding
+    # included) in one launch: every byte of the slot equals the source, NaN payloads and
+    # -0.0 included, and the forecasts then match those of per-layer pushes bit for bit.
+    eb = 2 if dt == bc.DTYPE_BF16 else 4
+    numels = [3 * 8192 + 3, 0, 16384 // eb * 5, 3, 100_003, 1]
+    h = bc.bc_cache_create(numels, 3, dt)
+    ref = bc.bc_cache_create(numels, 3, dt)
+    bc.bc_cache_set_kernel(h, kernel)
+    bc.bc_cache_set_kernel(ref, kernel)
+    try:
+        offs = bc.bc_cache_layout(h)
+        rng = np.random.default_rng(41)
+        images = []
+        for k in range(3):
+            if dt == bc.DTYPE_BF16:         # any bit pattern, specials planted up front
+                bits = rng.integers(0, 2 ** 16, offs[-1] // 2, dtype=np.uint16)
+                bits[:4] = [0x7FC1, 0xFFFF, 0x8000, 0x7F80]
+                images.append(to_device(bits))
+            else:                           # finite values except the planted specials
+                v = rng.standard_normal(offs[-1] // 4).astype(np.float32)
+                v.view(np.uint32)[:3] = [0x7FC00001, 0xFFFFFFFF, 0x80000000]
+                images.append(to_device(v))
+        times = [0.9, 0.85, 0.8]
+        p0 = bc.bc_cache_stats(h)
+        for k, t in enumerate(times):
+            bc.bc_cache_push_flat(h, images[k].data_ptr(), t, stream())
+            bc.bc_cache_push(ref, [images[k].data_ptr() + offs[l] if n else 0
+                                   for l, n in enumerate(numels)], t, stream())
+        torch.cuda.synchronize()
+        bc.bc_cache_check(h)
+        p1 = bc.bc_cache_stats(h)
+        assert p1["kernel_launches"] - p0["kernel_launches"] == 3
+        assert p1["pipeline_launches"] - p0["pipeline_launches"] == \
+            (3 if kernel == bc.KERNEL_PIPELINE else 0)
+        assert p1["table_uploads"] == p0["table_uploads"]
+        assert bc.bc_cache_nodes(h) == [0.8, 0.85, 0.9]
+        for j in range(3):
+            base = bc.bc_cache_slot_ptrs(h, j)[0]
+            whole = device_view(base, offs[-1] // eb, dt)
+            want = images[2 - j]
+            if dt == bc.DTYPE_F32:
+                assert torch.equal(whole.view(torch.int32), want.view(torch.int32))
+            else:
+                assert torch.equal(whole, want)
+        outs = {c: [empty_out(n, dt) for n in numels] for c in (h, ref)}
+        for c in (h, ref):
+            bc.bc_forecast(c, 0.75, [o.data_ptr() if n else None
+                                     for o, n in zip(outs[c], numels)], dt, stream())
+        torch.cuda.synchronize()
+        for a, b, n in zip(outs[h], outs[ref], numels):
+            if dt == bc.DTYPE_F32:
+                assert torch.equal(a[:n].view(torch.int32), b[:n].view(torch.int32))
+            else:
+                assert torch.equal(a[:n], b[:n])
+    finally:
+        bc.bc_cache_destroy(h)
+        bc.bc_cache_destroy(ref)
+
+
 def test_null_outputs_skip_layers_and_window_forecast():
     numels = [8192 * 3, 1000, 77_777, 64]
     times = [0.9, 0.8, 0.7]
