@@ -8,6 +8,10 @@
  *                       full-step features, forecast, read back, and compare every element
  *                       with the fp64 oracle (liboracle, linked for the check only); then
  *                       the probe drift of the two newest slots against the oracle's
+ *   abi_client manylayers 2048 ragged tensors: pushes and a forecast of one launch each
+ *                       through the device layer tables (oracle on every element, a planted
+ *                       NaN), then the same history as slot images through bc_cache_push_flat
+ *                       and bc_forecast_flat, bit for bit the per-layer forecast
  *
  * Exit status 0 on success; a failing check prints what failed and exits 1.
  */
@@ -171,6 +175,57 @@ static int device_checks(void) {
 /* A blockwise-style cache of 2048 ragged bf16 tensors: pushes and the forecast each run as
  * one launch (the layer tables travel through the handle's device copies), every element of
  * every tensor matches the oracle, and a NaN planted in one stored value comes out as NaN. */
+/* The same history pushed as slot images (bc_cache_push_flat) into a second cache and
+ * forecast into one slot-shaped output (bc_forecast_flat): one launch each and no layer
+ * table, bit for bit the per-layer forecast `want` (laid out at `offs`). */
+static int flat_slot_checks(const int64_t *numels, int L, const int64_t *offs,
+                            uint16_t *const *host, const double *times, double t_new,
+                            const uint16_t *want) {
+    int failures = 0;
+    bc_handle h = NULL;
+    int64_t *lay = (int64_t *)malloc((size_t)(L + 1) * sizeof(int64_t));
+    CHECK(bc_cache_create(numels, L, 3, BC_DTYPE_BF16, NULL, &h) == BC_OK, "create: %s",
+          bc_last_error());
+    CHECK(bc_cache_layout(h, lay) == BC_OK, "layout");
+    if (failures) return failures;
+    const size_t slot_bytes = (size_t)lay[L];
+    uint16_t *img = (uint16_t *)calloc(slot_bytes / 2, sizeof(uint16_t));
+    uint16_t *flat = (uint16_t *)malloc(slot_bytes);
+    void *dev_img = NULL, *dev_flat = NULL;
+    CHECK(cudaMalloc(&dev_img, slot_bytes) == 0 && cudaMalloc(&dev_flat, slot_bytes) == 0,
+          "cudaMalloc");
+    bc_stats st0, st1;
+    CHECK(bc_cache_stats(h, &st0) == BC_OK, "stats");
+    for (int k = 0; k < 3 && !failures; ++k) {
+        for (int l = 0; l < L; ++l)
+            memcpy(img + lay[l] / 2, host[k] + offs[l], (size_t)numels[l] * 2);
+        CHECK(cudaMemcpy(dev_img, img, slot_bytes, H2D) == 0, "upload");
+        CHECK(bc_cache_push_flat(h, dev_img, times[k], NULL) == BC_OK, "push_flat: %s",
+              bc_last_error());
+        cudaDeviceSynchronize();
+    }
+    CHECK(bc_forecast_flat(h, t_new, dev_flat, NULL) == BC_OK, "forecast_flat: %s",
+          bc_last_error());
+    CHECK(bc_cache_check(h) == BC_OK, "device status");
+    CHECK(bc_cache_stats(h, &st1) == BC_OK, "stats");
+    CHECK(st1.kernel_launches - st0.kernel_launches == 4, "%lld launches for 3 flat pushes "
+          "and a flat forecast", (long long)(st1.kernel_launches - st0.kernel_launches));
+    CHECK(st1.table_uploads == st0.table_uploads, "the flat calls uploaded a layer table");
+    CHECK(cudaMemcpy(flat, dev_flat, slot_bytes, D2H) == 0, "download");
+    int64_t diff = 0;
+    for (int l = 0; l < L && !failures; ++l)
+        for (int64_t e = 0; e < numels[l]; ++e)
+            if (flat[lay[l] / 2 + e] != want[offs[l] + e]) ++diff;
+    CHECK(diff == 0, "%lld flat elements differ from the per-layer forecast", (long long)diff);
+    bc_cache_destroy(h);
+    cudaFree(dev_img);
+    cudaFree(dev_flat);
+    free(img);
+    free(flat);
+    free(lay);
+    return failures;
+}
+
 static int many_layer_checks(void) {
     enum { L = 2048 };
     const double times[3] = {0.9, 0.85, 0.8};
@@ -249,6 +304,7 @@ static int many_layer_checks(void) {
         }
     }
     CHECK(bad == 0, "%lld elements off the oracle", (long long)bad);
+    if (!failures) failures += flat_slot_checks(numels, L, offs, host, times, t_new, got);
     bc_cache_destroy(h);
     cudaFree(dev_in);
     cudaFree(dev_out);
