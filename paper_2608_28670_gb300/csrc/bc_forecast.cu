@@ -197,14 +197,30 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
     a.inject = opt.inject;
     a.slot[0] = opt.dst_base;
     // The bulk-copy pipeline needs enough of its 32 KiB tiles per SM to amortise its ring.
+    // The layer table is filled with the tile shape of the kernel in question and filled
+    // again only if the choice falls on the register copy.
     a.n_layers = n;
     const int sms = sm_count();
+    constexpr int kPipeGroups = kCopyTileBytes / 16, kRegGroups = kThreads * kCopyVecsPerThread;
+    const bool forced = opt.kernel == BC_KERNEL_PIPELINE || opt.inject;
+    const bool weigh = !forced && opt.kernel == BC_KERNEL_AUTO;
+    LayerEntry *tab;
+    if constexpr (CAP == 0) {
+        std::vector<LayerEntry> &v = table_scratch();
+        v.resize(static_cast<size_t>(n));
+        tab = v.data();
+    } else {
+        tab = a.layer;
+    }
+    int tile_groups = forced || weigh ? kPipeGroups : kRegGroups;
+    a.total_tiles = fill_entries(tab, layers, n, T::kBytes, 16, tile_groups);
     const bool pipeline =
-        opt.kernel == BC_KERNEL_PIPELINE || opt.inject ||
-        (opt.kernel == BC_KERNEL_AUTO &&
-         count_tiles(layers, n, T::kBytes, kCopyTileBytes / kVecBytes) >=
-             static_cast<int64_t>(kCopyMinTilesPerCta) * sms);
-    const int tile_groups = pipeline ? kCopyTileBytes / 16 : kThreads * kCopyVecsPerThread;
+        forced || (weigh && a.total_tiles >= static_cast<int64_t>(kCopyMinTilesPerCta) * sms);
+    if (!pipeline && tile_groups != kRegGroups) {
+        tile_groups = kRegGroups;
+        a.total_tiles = fill_entries(tab, layers, n, T::kBytes, 16, tile_groups);
+    }
+    if (a.total_tiles == 0) return cudaSuccess;
     // the launch's error, after recording that a device-table launch reads its table
     auto launched = [&](cudaError_t e) -> int {
         if constexpr (CAP == 0) {
@@ -214,20 +230,13 @@ int copy_group(const LayerEntry *layers, int n, const CopyOptions &opt, cudaStre
         return e;
     };
     if constexpr (CAP == 0) {
-        std::vector<LayerEntry> &tab = table_scratch();
-        tab.resize(static_cast<size_t>(n));
-        a.total_tiles = fill_entries(tab.data(), layers, n, T::kBytes, 16, tile_groups);
-        if (a.total_tiles == 0) return cudaSuccess;
-        const int err = upload_table(*opt.table, tab.data(), n, s);
+        const int err = upload_table(*opt.table, tab, n, s);
         if (err != cudaSuccess) return err;
         a.table = opt.table->dev;
         if (pipeline) {
             const int64_t cap = static_cast<int64_t>(sms) * BC_COPY_CTAS_PER_SM;
-            fill_starts(a, tab.data(), n, a.total_tiles < cap ? a.total_tiles : cap);
+            fill_starts(a, tab, n, a.total_tiles < cap ? a.total_tiles : cap);
         }
-    } else {
-        a.total_tiles = fill_entries(a.layer, layers, n, T::kBytes, 16, tile_groups);
-        if (a.total_tiles == 0) return cudaSuccess;
     }
     if (pipeline) {
         auto kern = copy_tma_kernel<T, CAP>;

@@ -695,20 +695,14 @@ int resident_ctas(KernelPtr kern, std::atomic<int> &cache, int cap) {
     return c;
 }
 
-// Tiles of all layers for a tile of `tile_vecs` vectors.
-inline int64_t count_tiles(const LayerEntry *layers, int n, int elem_bytes, int tile_vecs) {
-    int64_t tiles = 0;
-    for (int i = 0; i < n; ++i) tiles += tiles_for(layers[i].numel, elem_bytes, kVecBytes, tile_vecs);
-    return tiles;
-}
-
 // Copy the layers into `dst` with their tile prefix sums; returns the number of tiles.
 inline int64_t fill_entries(LayerEntry *dst, const LayerEntry *layers, int n, int elem_bytes,
                             int vec_bytes, int tile_vecs) {
+    const TileCounter tiles_of(elem_bytes, vec_bytes, tile_vecs);
     int64_t tiles = 0;
     for (int i = 0; i < n; ++i) {
         dst[i] = layers[i];
-        tiles += tiles_for(layers[i].numel, elem_bytes, vec_bytes, tile_vecs);
+        tiles += tiles_of(layers[i].numel);
         dst[i].tile_end = tiles;
     }
     return tiles;
@@ -760,18 +754,26 @@ inline int table_used(DeviceTable &tb, cudaStream_t s) {
 }
 
 // Fill a.start[] with the layer of every CTA's first tile (contiguous ranges of
-// ceil(total / grid) tiles), as the kernels would find it.
+// ceil(total / grid) tiles), as the kernels would find it: the first layer whose tiles reach
+// past that tile (the last layer if none does), by binary search over the prefix sums, so
+// that tables of many thousands of layers are not walked once more per call.
 template <int CAP>
 inline void fill_starts(ForecastArgs<CAP> &a, const LayerEntry *tab, int n, int64_t grid) {
     a.n_starts = 0;
     if (grid > kMaxStartCtas || grid < 1) return;
     const int64_t per_cta = (a.total_tiles + grid - 1) / grid;
-    int l = 0;
     for (int64_t c = 0; c < grid; ++c) {
         const int64_t t = c * per_cta;
-        while (l < n - 1 && t >= tab[l].tile_end) ++l;
-        a.start[c].layer = l;
-        a.start[c].first = l > 0 ? tab[l - 1].tile_end : 0;
+        int lo = 0, hi = n - 1;
+        while (lo < hi) {
+            const int mid = lo + (hi - lo) / 2;
+            if (tab[mid].tile_end > t)
+                hi = mid;
+            else
+                lo = mid + 1;
+        }
+        a.start[c].layer = lo;
+        a.start[c].first = lo > 0 ? tab[lo - 1].tile_end : 0;
     }
     a.n_starts = static_cast<int32_t>(grid);
 }
@@ -807,21 +809,38 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
     // Kernel choice.  The pipeline kernel needs enough tiles per CTA to amortise filling its
     // ring; small launches (few or tiny layers) run the register kernel, and launches of
     // under BC_SMALL_LAUNCH_TILES_PER_SM of its tiles per SM use half-size tiles so that more
-    // SMs and threads share the few round trips.
+    // SMs and threads share the few round trips.  The layer table is filled (tile prefix
+    // sums) with the tile shape of the kernel in question and filled again only when the
+    // choice falls on another shape (at H <= 3 both kernels share one).
     constexpr int kRegVpt = kVecsPerThreadFor<K>;
-    const bool pipe_ok = K <= 3 || BC_TMA_AUTO_K4;
-    bool pipeline = p.kernel == BC_KERNEL_PIPELINE || p.inject;
-    if (!pipeline && p.kernel == BC_KERNEL_AUTO && pipe_ok) {
-        const int64_t tiles = count_tiles(layers, n, TIn::kBytes, kThreads * kTmaVpt<K>);
-        pipeline = tiles >= static_cast<int64_t>(kTmaMinTilesPerCta) * sms &&
-                   tiles >= static_cast<int64_t>(BC_TMA_MIN_TILES_PER_LAYER) * n;
+    constexpr int kTmaTile = kThreads * kTmaVpt<K>, kRegTile = kThreads * kRegVpt;
+    const bool forced = p.kernel == BC_KERNEL_PIPELINE || p.inject;
+    const bool weigh = !forced && p.kernel == BC_KERNEL_AUTO && (K <= 3 || BC_TMA_AUTO_K4);
+    LayerEntry *tab;
+    if constexpr (CAP == 0) {
+        std::vector<LayerEntry> &v = table_scratch();
+        v.resize(static_cast<size_t>(n));
+        tab = v.data();
+    } else {
+        tab = a.layer;
     }
-    int vpt = kRegVpt;
+    int tile_vecs = forced || weigh ? kTmaTile : kRegTile;
+    a.total_tiles = fill_entries(tab, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
+    bool pipeline = forced;
+    if (weigh)
+        pipeline = a.total_tiles >= static_cast<int64_t>(kTmaMinTilesPerCta) * sms &&
+                   a.total_tiles >= static_cast<int64_t>(BC_TMA_MIN_TILES_PER_LAYER) * n;
+    if (!pipeline && tile_vecs != kRegTile) {
+        tile_vecs = kRegTile;
+        a.total_tiles = fill_entries(tab, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
+    }
     if (!pipeline && CAP == kLayersSmall && p.kernel == BC_KERNEL_AUTO && kRegVpt > 1 &&
-        count_tiles(layers, n, TIn::kBytes, kThreads * kRegVpt) <
-            static_cast<int64_t>(BC_SMALL_LAUNCH_TILES_PER_SM) * sms)
-        vpt = 1;
-    const int tile_vecs = kThreads * (pipeline ? kTmaVpt<K> : vpt);
+        a.total_tiles < static_cast<int64_t>(BC_SMALL_LAUNCH_TILES_PER_SM) * sms) {
+        tile_vecs = kThreads;
+        a.total_tiles = fill_entries(tab, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
+    }
+    const int vpt = tile_vecs / kThreads;
+    if (a.total_tiles == 0) return cudaSuccess;
     // the launch's error, after recording that a device-table launch reads its table
     auto launched = [&](cudaError_t e) -> int {
         if constexpr (CAP == 0) {
@@ -832,11 +851,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
     };
 
     if constexpr (CAP == 0) {
-        std::vector<LayerEntry> &tab = table_scratch();
-        tab.resize(static_cast<size_t>(n));
-        a.total_tiles = fill_entries(tab.data(), layers, n, TIn::kBytes, kVecBytes, tile_vecs);
-        if (a.total_tiles == 0) return cudaSuccess;
-        const int err = upload_table(*p.table, tab.data(), n, s);
+        const int err = upload_table(*p.table, tab, n, s);
         if (err != cudaSuccess) return err;
         a.table = p.table->dev;
         // every CTA's first layer, as the kernels would find it (grid as launched below)
@@ -846,10 +861,7 @@ int launch_group(const LaunchPlan &p, const LayerEntry *layers, int n, int euler
             grid_cap *= resident_ctas(forecast_kernel<K, kRegVpt, TIn, TOut, 0>, occ_reg,
                                       BC_CTAS_PER_SM);
         }
-        fill_starts(a, tab.data(), n, a.total_tiles < grid_cap ? a.total_tiles : grid_cap);
-    } else {
-        a.total_tiles = fill_entries(a.layer, layers, n, TIn::kBytes, kVecBytes, tile_vecs);
-        if (a.total_tiles == 0) return cudaSuccess;
+        fill_starts(a, tab, n, a.total_tiles < grid_cap ? a.total_tiles : grid_cap);
     }
 
     if (pipeline) {

@@ -165,11 +165,25 @@ inline void kernel_weights(const double *c, int m, float *w, float *scale) {
 }
 
 // Tiles needed for `numel` elements of `elem_bytes` each, in vectors of `vec_bytes`,
-// `tile_vecs` vectors per tile.
+// `tile_vecs` vectors per tile: ceil(numel / (vec_bytes / elem_bytes * tile_vecs)) (the
+// vectors a layer needs, rounded up to whole tiles).  The table builders count many layers
+// with one tile shape; every shipped shape holds a power of two of elements, so the count is
+// a shift rather than a 64-bit division per layer.
+struct TileCounter {
+    int64_t per_tile;  // elements per tile
+    int shift = -1;    // log2(per_tile) when it is a power of two
+    TileCounter(int elem_bytes, int vec_bytes, int tile_vecs)
+        : per_tile(static_cast<int64_t>(vec_bytes / elem_bytes) * tile_vecs) {
+        if ((per_tile & (per_tile - 1)) == 0)
+            for (shift = 0; (int64_t{1} << shift) < per_tile; ++shift) {
+            }
+    }
+    int64_t operator()(int64_t numel) const {
+        return shift >= 0 ? (numel + per_tile - 1) >> shift : (numel + per_tile - 1) / per_tile;
+    }
+};
 inline int64_t tiles_for(int64_t numel, int elem_bytes, int vec_bytes, int tile_vecs) {
-    const int64_t ev = vec_bytes / elem_bytes;
-    const int64_t vecs = (numel + ev - 1) / ev;
-    return (vecs + tile_vecs - 1) / tile_vecs;
+    return TileCounter(elem_bytes, vec_bytes, tile_vecs)(numel);
 }
 
 // Enqueue the grouped forecast: one launch, or with more than kLayersLarge layers and no

@@ -3,7 +3,9 @@
  *
  *   abi_client host     host-only calls (weights, footprints, schedules, errors): no GPU
  *   abi_client hostcost host time of bc_forecast calls on small caches of 1-64 layers
- *                       (launch included; the GPU work is tiny), one JSON line per size
+ *                       (launch included; the GPU work is tiny), and per tensor of
+ *                       forecasts and pushes over 4096 and 65,536 tensors, one JSON line per
+ *                       size
  *   abi_client device   one cache on the current GPU: allocate with cudaMalloc, push three
  *                       full-step features, forecast, read back, and compare every element
  *                       with the fp64 oracle (liboracle, linked for the check only); then
@@ -322,16 +324,20 @@ static double now_s(void) {
 }
 
 /* Host cost of one forecast call through the ABI (memo hit, table build, launch), on
- * caches of 1, 4, 16 and 64 layers of 4096 bf16 elements, and of one memo lookup. */
+ * caches of 1, 4, 16 and 64 layers of 4096 bf16 elements, and of one memo lookup; then the
+ * host cost per tensor of forecasts and pushes over 4096 and 65,536 such tensors (device
+ * layer tables, reused each call). */
 static int host_cost(void) {
-    enum { kMaxLayers = 64, kCalls = 500, kElems = 4096 };
+    enum { kMaxLayers = 65536, kCalls = 500, kElems = 4096 };
+    static const int sizes[] = {1, 4, 16, 64, 4096, 65536};
     void *src = NULL, *out = NULL;
     CHECK(cudaMalloc(&src, kElems * 2) == 0 && cudaMalloc(&out, (size_t)kMaxLayers * kElems * 2) == 0,
           "cudaMalloc");
-    for (int L = 1; L <= kMaxLayers && !failures; L *= 4) {
-        int64_t numels[kMaxLayers];
-        const void *ptrs[kMaxLayers];
-        void *outs[kMaxLayers];
+    int64_t *numels = (int64_t *)malloc(sizeof(int64_t) * kMaxLayers);
+    const void **ptrs = (const void **)malloc(sizeof(void *) * kMaxLayers);
+    void **outs = (void **)malloc(sizeof(void *) * kMaxLayers);
+    for (size_t si = 0; si < sizeof sizes / sizeof sizes[0] && !failures; ++si) {
+        const int L = sizes[si];
         for (int l = 0; l < L; ++l) {
             numels[l] = kElems;
             ptrs[l] = src;
@@ -339,12 +345,15 @@ static int host_cost(void) {
         }
         bc_handle h = NULL;
         CHECK(bc_cache_create(numels, L, 3, BC_DTYPE_BF16, NULL, &h) == BC_OK, "create");
-        const double ts[3] = {0.9, 0.85, 0.8};
-        for (int k = 0; k < 3; ++k) CHECK(bc_cache_push(h, ptrs, ts[k], NULL) == BC_OK, "push");
-        for (int i = 0; i < 100; ++i) bc_forecast(h, 0.75, outs, BC_DTYPE_BF16, NULL);
+        if (failures) break;
+        double t = 0.9;
+        for (int k = 0; k < 3; ++k, t -= 0.05)
+            CHECK(bc_cache_push(h, ptrs, t, NULL) == BC_OK, "push");
+        const int calls = L > 64 ? 50 : kCalls;
+        for (int i = 0; i < 20; ++i) bc_forecast(h, 0.75, outs, BC_DTYPE_BF16, NULL);
         cudaDeviceSynchronize();
         const double t0 = now_s();
-        for (int i = 0; i < kCalls; ++i)
+        for (int i = 0; i < calls; ++i)
             CHECK(bc_forecast(h, 0.75, outs, BC_DTYPE_BF16, NULL) == BC_OK, "forecast");
         const double t1 = now_s();
         cudaDeviceSynchronize();
@@ -352,14 +361,25 @@ static int host_cost(void) {
         double c[BC_MAX_K];
         int m = 0;
         const double t3 = now_s();
-        for (int i = 0; i < kCalls; ++i) bc_coefficients(h, 0.75, c, &m);
+        for (int i = 0; i < calls; ++i) bc_coefficients(h, 0.75, c, &m);
         const double t4 = now_s();
+        const double t5 = now_s();
+        for (int i = 0; i < calls; ++i, t -= 1e-4)
+            CHECK(bc_cache_push(h, ptrs, t, NULL) == BC_OK, "push");
+        const double t6 = now_s();
+        cudaDeviceSynchronize();
         CHECK(bc_cache_check(h) == BC_OK, "device status");
         printf("{\"layers\": %d, \"host_us_per_forecast\": %.2f, \"device_us_per_forecast\": %.2f, "
-               "\"memo_lookup_us\": %.3f}\n", L, 1e6 * (t1 - t0) / kCalls,
-               1e6 * (t2 - t0) / kCalls, 1e6 * (t4 - t3) / kCalls);
+               "\"memo_lookup_us\": %.3f, \"host_us_per_push\": %.2f, "
+               "\"host_ns_per_tensor_forecast\": %.2f, \"host_ns_per_tensor_push\": %.2f}\n",
+               L, 1e6 * (t1 - t0) / calls, 1e6 * (t2 - t0) / calls, 1e6 * (t4 - t3) / calls,
+               1e6 * (t6 - t5) / calls, 1e9 * (t1 - t0) / calls / L,
+               1e9 * (t6 - t5) / calls / L);
         bc_cache_destroy(h);
     }
+    free(numels);
+    free(ptrs);
+    free(outs);
     cudaFree(src);
     cudaFree(out);
     return failures;

@@ -54,5 +54,10 @@ def test_c_client_host_cost_mode_runs(client):
     p = subprocess.run([client, "hostcost"], capture_output=True, text=True, timeout=300)
     assert p.returncode == 0, p.stdout + p.stderr
     rows = [json.loads(l) for l in p.stdout.splitlines() if l.startswith("{")]
-    assert [r["layers"] for r in rows] == [1, 4, 16, 64]
-    assert all(0 < r["host_us_per_forecast"] < 1000 and r["memo_lookup_us"] > 0 for r in rows)
+    assert [r["layers"] for r in rows] == [1, 4, 16, 64, 4096, 65536]
+    small, large = rows[:4], rows[4:]
+    assert all(0 < r["host_us_per_forecast"] < 1000 and r["memo_lookup_us"] > 0 for r in small)
+    # thousands of tensors: the per-call work is linear in the tensor count, well under a
+    # microsecond per tensor
+    assert all(0 < r["host_ns_per_tensor_forecast"] < 200 and 0 < r["host_ns_per_tensor_push"] < 200
+               for r in large)
