@@ -235,10 +235,10 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  * layers the launch reads its layer table from the handle's device copy, which is
  * re-uploaded (one cudaMemcpyAsync on `stream`, from pinned memory) only when the outputs
  * differ from the previous such call; the host waits only if four uploads of different
- * tables are still queued ahead of the device.  Such a call on another stream than the
- * previous one first makes `stream` wait (cudaStreamWaitEvent) for the previous launch that
- * read the table, so forecasts of one handle on several streams never see each other's
- * tables (their outputs remain the caller's to keep apart).  While `stream` is being
+ * tables are still queued ahead of the device.  Such a call first makes `stream` wait
+ * (cudaStreamWaitEvent) for the previous launch that read the table, so forecasts of one
+ * handle on several streams never see each other's tables (their outputs remain the
+ * caller's to keep apart).  While `stream` is being
  * captured into a CUDA graph it issues one launch per 1016 layers instead, so that the
  * graph holds its own tables.
  * Layers with a NULL output are skipped, which also serves to forecast a window of layers.

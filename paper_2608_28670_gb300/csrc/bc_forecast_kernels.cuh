@@ -711,12 +711,14 @@ inline int64_t fill_entries(LayerEntry *dst, const LayerEntry *layers, int n, in
 // Make the handle's device table hold `entries[0..n)` for a launch on `s`: one
 // cudaMemcpyAsync on `s` from the next pinned staging buffer, skipped when the previous upload
 // was the same table.  A staging buffer is rewritten only after the copy that last read it has
-// run (its event).  When the last launch that read the table went to another stream, `s`
-// first waits for it: that launch may still be reading the table this copy overwrites, and
-// a launch that reuses the table must follow the copy queued on that stream ahead of it.
+// run (its event).  `s` first waits for the last launch that read the table, whatever stream
+// it went to (on that same stream the wait is already met): that launch may still be reading
+// the table this copy overwrites, and a launch that reuses the table must follow the copy
+// queued ahead of it.  Stream handles are not compared, since a destroyed stream's handle can
+// come back as a new stream.
 inline int upload_table(DeviceTable &tb, const LayerEntry *entries, int n, cudaStream_t s) {
     const size_t bytes = sizeof(LayerEntry) * static_cast<size_t>(n);
-    if (tb.used_recorded && tb.used_stream != static_cast<void *>(s)) {
+    if (tb.used_recorded) {
         const cudaError_t e = cudaStreamWaitEvent(s, static_cast<cudaEvent_t>(tb.used), 0);
         if (e != cudaSuccess) return e;
     }
@@ -748,7 +750,6 @@ inline int upload_table(DeviceTable &tb, const LayerEntry *entries, int n, cudaS
 inline int table_used(DeviceTable &tb, cudaStream_t s) {
     const cudaError_t e = cudaEventRecord(static_cast<cudaEvent_t>(tb.used), s);
     if (e != cudaSuccess) return e;
-    tb.used_stream = s;
     tb.used_recorded = true;
     return cudaSuccess;
 }

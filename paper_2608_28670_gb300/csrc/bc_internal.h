@@ -105,7 +105,7 @@ static_assert(sizeof(ForecastArgs<kLayersLarge>) <= 32764, "layer table exceeds 
 // pinned staging is a ring of kTableStaging buffers, each reused only after the copy that
 // last read it has run (its event), so the host waits only if that many uploads with
 // different tables are still queued ahead of the device.  An event recorded after every
-// launch that reads the table lets a call on another stream wait (on the device) until that
+// launch that reads the table makes the next call's stream wait (on the device) until that
 // launch is done, before it rewrites the table or reads the copy queued ahead of it.
 constexpr int kTableStaging = 4;
 struct DeviceTable {
@@ -117,7 +117,6 @@ struct DeviceTable {
     bool pending[kTableStaging] = {};        // an event was recorded after the buffer's copy
     void *uploaded[kTableStaging] = {};      // cudaEvent_t per staging buffer
     void *used = nullptr;          // cudaEvent_t recorded after the last launch that read `dev`
-    void *used_stream = nullptr;   // that launch's stream
     bool used_recorded = false;
     int64_t uploads = 0;           // uploads so far
 };
