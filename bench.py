@@ -1283,6 +1283,22 @@ def _time_oracle(chunks, W, seconds):
     return done, spent
 
 
+def host_info():
+    """The host the CPU legs ran on: architecture, CPU model (lscpu, when present) and the
+    number of online cores."""
+    import platform
+    info = {"machine": platform.machine(), "nproc": os.cpu_count()}
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            key, _, val = line.partition(":")
+            if key.strip() in ("Model name", "Vendor ID", "Socket(s)", "NUMA node(s)"):
+                info[key.strip()] = val.strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return info
+
+
 def cpu_baseline_from_device(run, seconds):
     """The fp64 oracle on the host over a bounded sample of the same workload: 64 chunks of
     4 Mi consecutive elements of the live history slots (copied to the host first, outside
@@ -1323,14 +1339,20 @@ def cpu_baseline_from_device(run, seconds):
         cores = pool.workers
     finally:
         pool.close()
+    step_elems = run.w.layer_numel * run.n_feat
     return {"value": round(elems * per_elem / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
             "kind": "oracle", "elems_per_s": round(elems / secs, 1),
             "sample": f"{sample[0].size} elements ({n_chunks} chunks of "
                       f"{max(x.size for x in parts[0])} consecutive elements, "
                       f"layers round-robin) of the K={m} history slots, processed {1 + passes} "
                       f"times by {cores} spawned workers running the fp64 oracle, {secs:.1f} s",
+            "whole_step_s": round(step_elems / (elems / secs), 1),
+            "whole_step_s_is": f"extrapolated: the step's {step_elems} elements at the "
+                               f"sample's rate",
+            "host": host_info(),
             "single_core": {"value": round(n1 * per_elem / t1 / 1e9, 4), "cores": 1,
-                            "elems_per_s": round(n1 / t1, 1), "seconds": round(t1, 1)}}
+                            "elems_per_s": round(n1 / t1, 1), "seconds": round(t1, 1),
+                            "whole_step_s": round(step_elems / (n1 / t1), 1)}}
 
 
 GROUP_ELEMS = 1 << 27   # elements per node copied to the host at a time (full baselines)
@@ -1473,7 +1495,7 @@ def run_reference(args):
            "config": {"workload": w.name, "K": K, "nodes": list(p.nodes), "target": p.t,
                       "sample_elements_per_step": n},
            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores,
-                            "kind": "oracle", "sample": sample},
+                            "kind": "oracle", "sample": sample, "host": host_info()},
            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
