@@ -1054,12 +1054,25 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
         # at most 16 chunks: a cache of thousands of small tensors moves in spans, not in
         # thousands of copies and calls
         cl = run.window if run.window < run.n_feat else max(chunk_layers, -(-L // 16))
+        ring_mode = host_bytes < total
+        ring = int(host_bytes // max(sizes)) if ring_mode else 0
+        if ring_mode:
+            # chunks of a divisor of the ring, at most half of it: chunk c's layers take ring
+            # positions (c % regions) * cl onwards, so consecutive chunks use disjoint host
+            # buffers and one chunk's copies overlap the next one's (a ring of one layer
+            # leaves one chunk at a time)
+            limit = min(chunk_layers, ring // 2, run.window)
+            divisors = [d for d in range(1, limit + 1) if ring % d == 0]
+            cl = divisors[-1] if divisors else 1
         chunks = [list(range(c, min(c + cl, L))) for c in range(0, L, cl)]
+        regions = ring // cl if ring_mode else len(chunks)
+        region_of = [c % regions for c in range(len(chunks))]
+        pipelined = not ring_mode or ring >= 2
         s_in, s_fc, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         done_out = [None] * len(chunks)
+        done_region = [None] * regions      # last read-back out of each host region
         shared_outs = run.window < run.n_feat
 
-        ring_mode = host_bytes < total
         slot_offs = bc.bc_cache_layout(run.h, L)
 
         def out_of(l, ls):
@@ -1100,9 +1113,9 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
                 torch.from_numpy(host[offs[l0]:offs[l0] + n * eb]).view(tdt).copy_(
                     device_view(ptr, n, run.w.dtype).view(tdt), non_blocking=True)
 
-        def one_step_ring(i):
-            # Layers share host buffers: upload, forecast and read back one chunk at a time,
-            # in order on one stream, so no host buffer is read while it is being written.
+        def one_step_serial(i):
+            # A one-layer host ring: upload, forecast and read back one chunk at a time, in
+            # order on one stream, so no host buffer is read while it is being written.
             t_full, t_target = _continuation(run, i)
             slots = bc.bc_cache_next_slot_ptrs(run.h, L)
             bc.bc_cache_commit(run.h, t_full)
@@ -1116,9 +1129,41 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
                 ev.record(s_fc)
                 done_out[-1] = ev
 
+        def one_step_ring(i):
+            # Layers share host buffers: per chunk, the upload waits for the last read-back
+            # out of its host region (an earlier chunk of this step or the last step), then
+            # the forecast and the read-back follow on their own streams, so the next
+            # chunk's upload (another region) overlaps them.
+            t_full, t_target = _continuation(run, i)
+            slots = bc.bc_cache_next_slot_ptrs(run.h, L)
+            bc.bc_cache_commit(run.h, t_full)
+            for c, ls in enumerate(chunks):
+                g = region_of[c]
+                with torch.cuda.stream(s_in):
+                    if done_region[g] is not None:
+                        s_in.wait_event(done_region[g])
+                    h2d(c, slots)
+                    landed = torch.cuda.Event()
+                    landed.record(s_in)
+                s_fc.wait_event(landed)
+                if shared_outs:   # the window's output buffers are reused by every chunk
+                    prev = done_out[c - 1] if c > 0 else done_out[-1]
+                    if prev is not None:
+                        s_fc.wait_event(prev)
+                bc.bc_forecast(run.h, t_target, chunk_ptrs[c], run.out_dtype, s_fc.cuda_stream)
+                ev = torch.cuda.Event()
+                ev.record(s_fc)
+                with torch.cuda.stream(s_out):
+                    s_out.wait_event(ev)
+                    d2h(c)
+                    ev2 = torch.cuda.Event()
+                    ev2.record(s_out)
+                    done_out[c] = ev2
+                    done_region[g] = ev2
+
         def one_step(i):
             if ring_mode:
-                return one_step_ring(i)
+                return one_step_ring(i) if pipelined else one_step_serial(i)
             t_full, t_target = _continuation(run, i)
             slots = bc.bc_cache_next_slot_ptrs(run.h, L)
             landed = []
@@ -1159,7 +1204,7 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
         for i in range(steps):
             one_step(i + 1)
             ev = torch.cuda.Event(enable_timing=True)      # this step's last read-back
-            ev.record(s_fc if ring_mode else s_out)
+            ev.record(s_out if pipelined else s_fc)
             marks.append(ev)
         for ev in done_out:
             if ev is not None:
@@ -1182,10 +1227,13 @@ def e2e(run, steps, world, dist, chunk_layers=6, host_cap_bytes=48 * 10**9):
                                       if link and link.get("both_GB/s") else None),
                 "ms_per_step": round(ms, 3), "wall_s": round(wall, 3), "steps": steps,
                 "chunk_layers": cl, "host_memory": kind, "host_buffer_bytes": int(host_bytes),
-                "overlapped": not ring_mode,
+                "overlapped": pipelined,
+                "host_ring_layers": ring or None,
                 "path": "pinned host -> next cache slot (bc_cache_next_slot_ptrs + "
                         "bc_cache_commit) -> bc_forecast per chunk -> pinned host, " +
                         ("pipelined over 3 streams" if not ring_mode else
+                         f"pipelined over 3 streams through a ring of {ring} layers of host "
+                         "buffers (page-locked memory capped per rank)" if pipelined else
                          "one chunk at a time on one stream (host buffers shared by layers)")}
     finally:
         torch.cuda.synchronize()
