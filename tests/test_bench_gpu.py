@@ -40,3 +40,20 @@ def test_bench_line_keeps_the_contract():
     assert c["kind"] == "oracle" and c["cores"] >= 1 and c["value"] > 0 and c["sample"]
     if d["clocks"] is not None:
         assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(d["clocks"])
+
+
+def test_end_to_end_leg_pipelines_a_capped_host_ring():
+    # With less page-locked memory than one slot (a rank's share of a node's cap), the e2e
+    # leg cycles layers through a ring of host buffers and still overlaps the copies: the
+    # DiT-XL/2 512 px slot (28 layers of 18.9 MB) under a 0.2 GB cap is a ring of 10 layers,
+    # moved in chunks of 5, a whole slot each way per step.
+    p = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--workload", "c2i-512",
+                        "--steps", "3", "--warmup", "3", "--no-sweep", "--no-extra",
+                        "--no-cpu-baseline", "--no-clocks", "--e2e-host-cap-gb", "0.2"],
+                       capture_output=True, text=True, timeout=600)
+    assert p.returncode == 0, p.stderr[-3000:]
+    e = json.loads(p.stdout.strip().splitlines()[-1])["e2e"]
+    slot = 28 * 8 * 1024 * 1152 * 2
+    assert e["h2d_bytes_per_step"] == slot and e["d2h_bytes_per_step"] == slot
+    assert e["host_ring_layers"] == 10 and e["chunk_layers"] == 5 and e["overlapped"] is True
+    assert e["host_buffer_bytes"] == 10 * slot // 28 and e["value"] > 0
