@@ -14,7 +14,8 @@ def pytest_configure(config):
 
 def pytest_collection_modifyitems(config, items):
     # A GPU test on a machine without a GPU is skipped with a reason rather than erroring;
-    # on a GPU machine the library must load, so a missing build fails loudly inside the test.
+    # on a machine with a GPU the library must load, so a missing build fails loudly inside
+    # the test.
     if not any("gpu" in item.keywords for item in items):
         return
     try:
