@@ -96,12 +96,12 @@ typedef struct bc_cache *bc_handle;
 
 /* Kernel selection (bc_cache_set_kernel) for forecasts, probe drifts and push copies.
  * AUTO picks per launch:
- *  - forecast: the shared-memory pipeline (TMA bulk copies into a three-stage ring, one CTA
- *    per SM) for H <= 3 when the launch has at least 16 tiles of 8 Ki bf16 / 4 Ki fp32
- *    elements per SM, else the register kernel (each thread holds its history loads in
- *    registers; up to two CTAs per SM; half-size tiles when the launch has fewer than two
- *    tiles per SM); H = 4 uses the register kernel unless PIPELINE is pinned.  All forms
- *    compute the same bits.
+ *  - forecast: the shared-memory pipeline (TMA bulk copies into a ring, one CTA per SM:
+ *    three stages of 16 KiB per history slot at H <= 3, five of 8 KiB at H = 4) when the
+ *    launch has at least 16 of its tiles per SM and its layers average at least 32 tiles,
+ *    else the register kernel (each thread holds its history loads in registers; up to two
+ *    CTAs per SM; half-size tiles when the launch has fewer than two tiles per SM).  All
+ *    forms compute the same bits.
  *  - probe drift: the pipeline form (a five-stage ring of 16 KiB tiles of both tensors, one
  *    CTA per SM) from 16 such tiles per SM on, else register loads.  The two forms group
  *    the partial sums differently, so they agree within rounding, not bit for bit.
@@ -112,7 +112,7 @@ typedef enum { BC_KERNEL_AUTO = 0, BC_KERNEL_REGISTER = 1, BC_KERNEL_PIPELINE = 
 
 typedef struct {
     int64_t forecasts;       /* successful forecast calls (every bc_forecast* variant) */
-    int64_t pushes;          /* successful bc_cache_push / bc_cache_commit calls */
+    int64_t pushes;          /* successful bc_cache_push / _push_flat / _commit calls */
     int64_t kernel_launches; /* CUDA kernels this handle has launched */
     int64_t memo_hits;       /* Diff Key lookups answered from the memo (Eq. 7) */
     int64_t memo_misses;     /* Diff Key lookups that ran the solver */
@@ -158,8 +158,8 @@ bc_status bc_cache_bytes_for(const int64_t *numels, int n_layers, int K, bc_dtyp
  * bc_probe_drift plus a status word, and for caches of more than 1016 layers two layer
  * tables (forecast, push) of 32 bytes per layer in device memory, each with four times that
  * of pinned host staging (the only allocations the library makes; freed by
- * bc_cache_destroy).  p == NULL uses the paper's
- * defaults.  Blocks until the allocation is done.  Errors: INVALID_ARG, OOM, CUDA. */
+ * bc_cache_destroy).  p == NULL uses the paper's defaults.  Blocks until the allocation is
+ * done.  Errors: INVALID_ARG, OOM, CUDA. */
 bc_status bc_cache_create(const int64_t *numels, int n_layers, int K, bc_dtype dtype,
                           const bc_params *p, bc_handle *out);
 
@@ -238,9 +238,8 @@ bc_status bc_coefficients(bc_handle h, double t_new, double *c_out, int *m_out);
  * tables are still queued ahead of the device.  Such a call first makes `stream` wait
  * (cudaStreamWaitEvent) for the previous launch that read the table, so forecasts of one
  * handle on several streams never see each other's tables (their outputs remain the
- * caller's to keep apart).  While `stream` is being
- * captured into a CUDA graph it issues one launch per 1016 layers instead, so that the
- * graph holds its own tables.
+ * caller's to keep apart).  While `stream` is being captured into a CUDA graph it issues
+ * one launch per 1016 layers instead, so that the graph holds its own tables.
  * Layers with a NULL output are skipped, which also serves to forecast a window of layers.
  * Outputs must not overlap the arena (checked) or each other (not checked: overlapping
  * outputs race).
