@@ -19,7 +19,8 @@
 //   forecast_tma_kernel  TMA bulk copies into a shared-memory ring of stages, one CTA per
 //                        SM (H <= 3, and H = 4 with smaller tiles);
 //   forecast_kernel      every thread issues all of its 256-bit loads into registers before
-//                        using any, up to two CTAs per SM (H = 4, and small launches).
+//                        using any, up to two CTAs per SM (small launches, and many small
+//                        tensors).
 //
 // Arithmetic: the host divides the fp32 weights by a power of two `scale` >= sum_j |W_j|
 // (kernel_weights), the kernels accumulate in fp32 with FMA in node order j = 1..H and
