@@ -807,7 +807,9 @@ def time_blockwise(stream, steps):
 def time_other_workloads(stream, steps, cpu=False):
     """The remaining workloads: c2i-256 (9.4 MB per forecast, L2-resident, so L2 is flushed
     by writing 512 MB before every timed launch, outside its event pair; the flush keeps the
-    device busy while the host enqueues the forecast), c2i-512 (K = 4, 2.6 GB) and t2i-1024
+    device busy while the host enqueues the forecast; `us_after_clean_flush` adds a 512 MB
+    read after the write, so that no dirty line is left for the forecast to write back),
+    c2i-512 (K = 4, 2.6 GB) and t2i-1024
     (K = 3, 4.2 GB), whose inputs exceed L2: `steps` forecasts back to back between one event
     pair, as in the headline measurement.  `idle_start_us` is one call on an idle device
     (host call to completion: memo lookup, table build and launch latency included).  With
@@ -816,6 +818,7 @@ def time_other_workloads(stream, steps, cpu=False):
     from paper_2608_28670_gb300.configs import WORKLOADS
     from paper_2608_28670_gb300.runner import WorkloadRun
     flush = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda")
+    clean = torch.zeros(128 * 2**20, dtype=torch.int32, device="cuda")   # 512 MB, read only
     out = {}
 
     def pair():
@@ -827,7 +830,7 @@ def time_other_workloads(stream, steps, cpu=False):
         try:
             warm_up(lambda i: r.forecast(), 3)
             p0 = r.stats()["pipeline_launches"]
-            warm_us = None
+            warm_us = clean_us = floor_us = None
             if name == "c2i-256":
                 ms = []
                 for i in range(steps):
@@ -839,6 +842,33 @@ def time_other_workloads(stream, steps, cpu=False):
                     torch.cuda.synchronize()
                     ms.append(a.elapsed_time(b))
                 m = statistics.median(ms)
+                # the same after a flush that leaves L2 clean: the write, then a 512 MB read
+                # (both outside the events), so that the forecast reads its history from HBM
+                # without also writing back the flush's dirty lines it evicts
+                ms_clean = []
+                for i in range(steps):
+                    flush.fill_(i & 0xFF)
+                    clean.sum()
+                    a, b = pair()
+                    a.record()
+                    r.forecast()
+                    b.record()
+                    torch.cuda.synchronize()
+                    ms_clean.append(a.elapsed_time(b))
+                clean_us = round(1e3 * statistics.median(ms_clean), 1)
+                # the floor of that measurement: a one-element fill, timed the same way
+                tiny = torch.zeros(1, dtype=torch.int32, device="cuda")
+                ms_floor = []
+                for i in range(steps):
+                    flush.fill_(i & 0xFF)
+                    clean.sum()
+                    a, b = pair()
+                    a.record()
+                    tiny.fill_(i)
+                    b.record()
+                    torch.cuda.synchronize()
+                    ms_floor.append(a.elapsed_time(b))
+                floor_us = round(1e3 * statistics.median(ms_floor), 1)
                 # beside it: launches back to back with the 9.4 MB resident in L2, replayed
                 # from a CUDA graph so that the host's per-call cost is not what is timed
                 g = torch.cuda.CUDAGraph()
@@ -881,6 +911,8 @@ def time_other_workloads(stream, steps, cpu=False):
                          "elems_per_s": round(r.w.layer_numel * r.n_feat / (m * 1e-3), 1),
                          "idle_start_us": round(1e3 * statistics.median(idle), 1),
                          "l2_warm_back_to_back_us": warm_us,
+                         "us_after_clean_flush": clean_us,
+                         "one_element_kernel_us_after_clean_flush": floor_us,
                          "K": r.K, "pipeline_kernel": pipe > 0,
                          "cache_bytes": bc_cache_bytes(r),
                          "l2": "flushed before each launch" if name == "c2i-256"
