@@ -8,9 +8,10 @@
 // given device: (1) a persistent grid streams both tensors once in 16-byte groups, each
 // thread sums a group in fp32 and accumulates the group sums with compensated (Kahan) fp32
 // addition, so the error stays near two fp32 ulps however long the stream is, without
-// touching GB300's slow fp64 pipe per element; every CTA adds its threads' sums in fp64
-// and writes its two partial sums to scratch; (2) one CTA adds the partials in index order
-// and writes {sum |d|, sum |prev|, ratio}.  HBM-bound: 2 * n * sizeof(T) bytes, no atomics.
+// touching GB300's slow fp64 pipe per element; every CTA adds its threads' sums with a
+// fixed compensated fp32 shuffle tree, converts once per warp to fp64 and writes its two
+// partial sums to scratch; (2) one CTA adds the partials in a fixed order and writes
+// {sum |d|, sum |prev|, ratio}.  HBM-bound: 2 * n * sizeof(T) bytes, no atomics.
 // The first launch comes in two forms: drift_partials (register loads, four groups in
 // flight per thread, grid stride; small probes) and drift_tma_partials (one CTA per SM
 // streaming a contiguous range of tiles through a five-stage TMA ring in shared memory;
@@ -73,9 +74,6 @@ struct Kahan {
         c = (t - s) - y;
         s = t;
     }
-    __device__ __forceinline__ double value() const {
-        return static_cast<double>(s) - static_cast<double>(c);
-    }
 };
 
 // Sum |c - p| and |p| over one 16-byte group of each tensor (fp32, fixed order).
@@ -96,17 +94,93 @@ __device__ __forceinline__ void group_sums(uint4 rc, uint4 rp, float &gd, float 
 
 constexpr int kGroupsInFlight = 4;
 
-// Fixed-order tree sum of one double per thread over the CTA (kProbeThreads threads).
-__device__ __forceinline__ double block_sum(double v, double *sh) {
-    sh[threadIdx.x] = v;
-    __syncthreads();
-    for (int s = kProbeThreads / 2; s > 0; s >>= 1) {
-        if (static_cast<int>(threadIdx.x) < s) sh[threadIdx.x] += sh[threadIdx.x + s];
-        __syncthreads();
+// Fixed-order tree sums of two doubles per thread over the CTA (kProbeThreads threads):
+// a shuffle tree within each warp, then warp 0 sums the warps' results the same way, so
+// the order never changes (bitwise reproducible) and the CTA waits at three barriers, not
+// at one per tree level (the fp64 adds are on GB300's slow fp64 pipe, so every level is
+// latency on the critical path).  `sh` holds at least 2 x (kProbeThreads / 32) doubles.
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+    return v;  // lane 0
+}
+
+__device__ __forceinline__ void block_sum2(double &a, double &b, double *sh) {
+    constexpr int kWarps = kProbeThreads / 32;
+    const int w = static_cast<int>(threadIdx.x) / 32, lane = static_cast<int>(threadIdx.x) % 32;
+    a = warp_sum(a);
+    b = warp_sum(b);
+    if (lane == 0) {
+        sh[w] = a;
+        sh[kWarps + w] = b;
     }
-    const double r = sh[0];
     __syncthreads();
-    return r;
+    if (w == 0) {
+        double ra = lane < kWarps ? sh[lane] : 0.0;
+        double rb = lane < kWarps ? sh[kWarps + lane] : 0.0;
+        ra = warp_sum(ra);
+        rb = warp_sum(rb);
+        if (lane == 0) {
+            sh[0] = ra;
+            sh[1] = rb;
+        }
+    }
+    __syncthreads();
+    a = sh[0];
+    b = sh[1];
+    __syncthreads();  // `sh` may be written again right after
+}
+
+// A compensated fp32 value hi + lo.  Two of them add with Knuth's error-free TwoSum on the
+// high parts (the rounding error of hi_a + hi_b is recovered exactly) and a plain sum of the
+// low parts, so a tree of them keeps about twice fp32's precision on the fast fp32 pipe.
+struct F2 {
+    float hi, lo;
+};
+
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+    const float s = a.hi + b.hi;
+    const float bv = s - a.hi;
+    const float e = (a.hi - (s - bv)) + (b.hi - bv);
+    return {s, (a.lo + b.lo) + e};
+}
+
+__device__ __forceinline__ F2 warp_sum_f2(F2 v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const F2 u{__shfl_down_sync(0xffffffffu, v.hi, o), __shfl_down_sync(0xffffffffu, v.lo, o)};
+        v = f2_add(v, u);
+    }
+    return v;  // lane 0
+}
+
+// CTA sums of every thread's two Kahan accumulators, in a fixed order: a compensated fp32
+// shuffle tree within each warp, one conversion to fp64 per warp, and thread 0 adds the
+// warps' sums in warp order.  The results are valid in thread 0.  The only fp64 work is the
+// per-warp conversion and eight additions: GB300 issues about two fp64 operations per cycle
+// per SM, so a per-thread fp64 tree costs microseconds per launch.  `sh` holds at least
+// 2 x (kProbeThreads / 32) doubles.
+__device__ __forceinline__ void block_sum_kahan(const Kahan &a, const Kahan &b, double *sh,
+                                                double &ra, double &rb) {
+    constexpr int kWarps = kProbeThreads / 32;
+    const int w = static_cast<int>(threadIdx.x) / 32, lane = static_cast<int>(threadIdx.x) % 32;
+    const F2 va = warp_sum_f2({a.s, -a.c});  // a Kahan sum is s - c
+    const F2 vb = warp_sum_f2({b.s, -b.c});
+    if (lane == 0) {
+        sh[w] = static_cast<double>(va.hi) + static_cast<double>(va.lo);
+        sh[kWarps + w] = static_cast<double>(vb.hi) + static_cast<double>(vb.lo);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double sa = 0.0, sb = 0.0;
+        for (int i = 0; i < kWarps; ++i) {
+            sa += sh[i];
+            sb += sh[kWarps + i];
+        }
+        ra = sa;
+        rb = sb;
+    }
+    __syncthreads();  // `sh` may be written again right after
 }
 
 template <bool kBf16>
@@ -148,8 +222,8 @@ __global__ void __launch_bounds__(kProbeThreads)
             sp.add(fabsf(p));
         }
     }
-    const double bd = block_sum(sd.value(), sh);
-    const double bp = block_sum(sp.value(), sh);
+    double bd = 0.0, bp = 0.0;
+    block_sum_kahan(sd, sp, sh, bd, bp);
     if (threadIdx.x == 0) {
         partials[2 * blockIdx.x] = bd;
         partials[2 * blockIdx.x + 1] = bp;
@@ -252,8 +326,8 @@ __global__ void __launch_bounds__(kProbeThreads)
             sp.add(fabsf(p));
         }
     }
-    const double bd = block_sum(sd.value(), sh);
-    const double bp = block_sum(sp.value(), sh);
+    double bd = 0.0, bp = 0.0;
+    block_sum_kahan(sd, sp, sh, bd, bp);
     if (threadIdx.x == 0) {
         partials[2 * blockIdx.x] = bd;
         partials[2 * blockIdx.x + 1] = bp;
@@ -268,8 +342,7 @@ __global__ void __launch_bounds__(kProbeThreads)
         sd += partials[2 * i];
         sp += partials[2 * i + 1];
     }
-    sd = block_sum(sd, sh);
-    sp = block_sum(sp, sh);
+    block_sum2(sd, sp, sh);
     if (threadIdx.x == 0) {
         out[0] = sd;
         out[1] = sp;
@@ -349,7 +422,9 @@ int launch_drift(const void *cur, const void *prev, int64_t n, bc_dtype dtype, d
         if (err != cudaSuccess) return err;
         ++*pipeline_launches;
     } else {
-        int64_t want = (nvec + kProbeThreads - 1) / kProbeThreads;
+        // one CTA per kProbeThreads x kGroupsInFlight groups: no CTA without data
+        constexpr int64_t kCtaGroups = static_cast<int64_t>(kProbeThreads) * kGroupsInFlight;
+        int64_t want = (nvec + kCtaGroups - 1) / kCtaGroups;
         if (want < 1) want = 1;
         grid = probe_ctas();
         if (grid > max_parts) grid = max_parts;
@@ -431,8 +506,8 @@ __global__ void __launch_bounds__(kProbeThreads)
                 }
             }
         }
-        const double bd = block_sum(sd.value(), sh);
-        const double bp = block_sum(sp.value(), sh);
+        double bd = 0.0, bp = 0.0;
+        block_sum_kahan(sd, sp, sh, bd, bp);
         if (threadIdx.x == 0) {
             partials[2 * tile] = bd;
             partials[2 * tile + 1] = bp;
