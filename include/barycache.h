@@ -345,9 +345,9 @@ bc_status bc_adaptive_decide(bc_adaptive *s, double drift, int *run_full);
  * cur, prev: device, n elements of dtype, 16-byte aligned; out: 3 device doubles.  Two
  * launches on `stream` with a fixed reduction order (bitwise reproducible on one device for
  * a given kernel choice), using the handle's reduction scratch, so calls on one handle must
- * not overlap on the device.  If the pipeline form gives up waiting (see bc_cache_check), out[] reads NaN.  The
- * caller reads out[2] back to drive bc_adaptive_decide.  Errors: INVALID_ARG, ALIGNMENT,
- * CUDA. */
+ * not overlap on the device.  If the pipeline form gives up waiting (see bc_cache_check),
+ * out[] reads NaN.  The caller reads out[2] back to drive bc_adaptive_decide.  Errors:
+ * INVALID_ARG, ALIGNMENT, CUDA. */
 bc_status bc_probe_drift(bc_handle h, const void *cur, const void *prev, int64_t n,
                          bc_dtype dtype, double *out, void *stream);
 
