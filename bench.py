@@ -560,8 +560,28 @@ def time_probe(run, steps, probe_elems=None):
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / steps
     nbytes = 2 * n * run.w.elem_bytes
+    # a realistic adaptive-schedule probe is a few MB and latency-bound: the device time of
+    # one call on a DiT-XL/2 256 px block output's worth of elements (589,824 of the cache
+    # dtype), 100 calls replayed from a CUDA graph so that the host's per-call cost is not
+    # what is timed (the probe stays in L2 between calls)
+    small_n = min(589824, n)
+    g = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+            for _ in range(100):
+                bc.bc_probe_drift(run.h, cur, prev, small_n, run.w.dtype, out.data_ptr(),
+                                  side.cuda_stream)
+    g.replay()
+    torch.cuda.synchronize()
+    a.record()
+    g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    small_us = 1e3 * a.elapsed_time(b) / 100
     return {"GB/s": round(nbytes / (ms * 1e-3) / 1e9, 1), "ms": round(ms, 4),
             "elements": n, "bytes_per_call": nbytes, "drift": round(float(out[2].item()), 6),
+            "small_probe_us": round(small_us, 2), "small_probe_elements": small_n,
             "what": "bc_probe_drift over layer 0 (newest vs previous node)" if not probe_elems
                     else "bc_probe_drift over the first elements of the two newest slots"}
 
