@@ -106,3 +106,59 @@ def test_graph_replay_equals_eager_loop_and_oracle():
         bc.bc_cache_check(h)
     finally:
         bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE])
+def test_probe_drift_replays_from_a_graph(kernel):
+    # The adaptive schedule's probe drift (handle and no-allocation forms) enqueues kernels
+    # only, so it can be captured: a replay computes from the probe tensors' current contents,
+    # bit for bit the eager call on the same contents, and both match the fp64 oracle.
+    n = 600_001                                    # ragged: a tail shorter than one group
+    rng = np.random.default_rng(7)
+    prev_h = rng.standard_normal(n).astype(np.float32)
+    cur_h = prev_h + 0.05 * rng.standard_normal(n).astype(np.float32)
+    cur, prev = torch.from_numpy(cur_h).cuda(), torch.from_numpy(prev_h).cuda()
+    f64 = dict(dtype=torch.float64, device="cuda")
+    h = bc.bc_cache_create([16], 2, bc.DTYPE_F32)
+    bc.bc_cache_set_kernel(h, kernel)
+    s = torch.cuda.current_stream().cuda_stream
+
+    def eager():
+        o, o_na = torch.zeros(3, **f64), torch.zeros(3, **f64)
+        bc.bc_probe_drift(h, cur.data_ptr(), prev.data_ptr(), n, bc.DTYPE_F32, o.data_ptr(), s)
+        bc.bc_probe_drift_noalloc(cur.data_ptr(), prev.data_ptr(), n, bc.DTYPE_F32,
+                                  o_na.data_ptr(), s)
+        torch.cuda.synchronize()
+        return o, o_na
+
+    try:
+        e, e_na = eager()                          # also the first, uncaptured calls
+        out, out_na = torch.full((3,), -1.0, **f64), torch.full((3,), -1.0, **f64)
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        with torch.cuda.stream(side):
+            l0 = bc.bc_cache_stats(h)["kernel_launches"]
+            with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+                bc.bc_probe_drift(h, cur.data_ptr(), prev.data_ptr(), n, bc.DTYPE_F32,
+                                  out.data_ptr(), side.cuda_stream)
+                bc.bc_probe_drift_noalloc(cur.data_ptr(), prev.data_ptr(), n, bc.DTYPE_F32,
+                                          out_na.data_ptr(), side.cuda_stream)
+            assert bc.bc_cache_stats(h)["kernel_launches"] - l0 == 2
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(out, e) and torch.equal(out_na, e_na)
+        np.testing.assert_allclose(out.cpu().numpy(), oracle.drift(cur_h, prev_h), rtol=2e-6)
+        np.testing.assert_allclose(out_na.cpu().numpy(), oracle.drift(cur_h, prev_h), rtol=2e-6)
+        cur.mul_(2.0)                              # new contents: the replay must read them
+        cur_h = cur_h * np.float32(2.0)
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        e2, e2_na = eager()
+        assert torch.equal(out, e2) and torch.equal(out_na, e2_na)
+        assert not torch.equal(out, e)
+        np.testing.assert_allclose(out.cpu().numpy(), oracle.drift(cur_h, prev_h), rtol=2e-6)
+        bc.bc_cache_check(h)
+    finally:
+        torch.cuda.synchronize()
+        bc.bc_cache_destroy(h)
