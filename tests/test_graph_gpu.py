@@ -162,3 +162,48 @@ def test_probe_drift_replays_from_a_graph(kernel):
     finally:
         torch.cuda.synchronize()
         bc.bc_cache_destroy(h)
+
+
+@pytest.mark.parametrize("kernel", [bc.KERNEL_REGISTER, bc.KERNEL_PIPELINE])
+def test_pushes_replay_from_a_graph(kernel):
+    # A push over more layers than a parameter block holds (split into parameter-block launches
+    # while captured) and a flat push of a slot image, captured into one graph: each replay
+    # copies the sources' current bytes into the slots chosen while capturing.
+    n_l, n = 2048, 2048
+    K = 3
+    h = bc.bc_cache_create([n] * n_l, K, bc.DTYPE_BF16)
+    bc.bc_cache_set_kernel(h, kernel)
+    s = torch.cuda.current_stream().cuda_stream
+    try:
+        offs = bc.bc_cache_layout(h)
+        src = torch.randint(-32768, 32767, (n * n_l,), dtype=torch.int16, device="cuda")
+        img = torch.randint(-32768, 32767, (offs[-1] // 2,), dtype=torch.int16, device="cuda")
+        ptrs = np.array([src.data_ptr() + 2 * n * l for l in range(n_l)], dtype=np.uint64)
+        bc.bc_cache_push(h, ptrs, 0.9, s)          # first uses outside the capture
+        bc.bc_cache_push_flat(h, img.data_ptr(), 0.8, s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        with torch.cuda.stream(side):
+            l0 = bc.bc_cache_stats(h)["kernel_launches"]
+            with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+                bc.bc_cache_push(h, ptrs, 0.7, side.cuda_stream)
+                bc.bc_cache_push_flat(h, img.data_ptr(), 0.6, side.cuda_stream)
+            assert bc.bc_cache_stats(h)["kernel_launches"] - l0 == 4    # 1016 + 1016 + 16, 1
+        # slots chosen while capturing: 0.7 went to node 1's slot, 0.6 to node 0's
+        per_layer_slot = bc.bc_cache_slot_ptrs(h, 1)[0]
+        flat_slot = bc.bc_cache_slot_ptrs(h, 0)[0]
+        for _ in range(2):
+            src.add_(1)
+            img.sub_(3)
+            torch.cuda.synchronize()
+            g.replay()
+            torch.cuda.synchronize()
+            got = device_view(per_layer_slot, n * n_l, bc.DTYPE_BF16)
+            assert torch.equal(got, src)
+            got = device_view(flat_slot, offs[-1] // 2, bc.DTYPE_BF16)
+            assert torch.equal(got, img)
+        bc.bc_cache_check(h)
+    finally:
+        torch.cuda.synchronize()
+        bc.bc_cache_destroy(h)
