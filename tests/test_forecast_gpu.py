@@ -425,6 +425,34 @@ def test_many_layers_in_a_graph_carry_their_own_tables(kernel):
         bc.bc_cache_destroy(h)
 
 
+def test_queued_table_uploads_wait_for_their_staging_buffers():
+    # Forecasts over more layers than a parameter block holds upload their layer table through
+    # a ring of four pinned staging buffers.  Eight forecasts into eight different output sets,
+    # queued behind ~50 ms of device work, need eight uploads: the fifth and later ones must
+    # wait until the copies queued earlier have read their staging buffers, and every output
+    # set must come out exactly as from a forecast issued alone.
+    numels = [(i * 37) % 301 + 1 for i in range(1100)]
+    h = run_case(numels, 2, 2, bc.DTYPE_F32, bc.DTYPE_BF16, bc.make_params(), 0.8, [0.9, 0.85],
+                 seed=9)
+    try:
+        ref = [empty_out(n, bc.DTYPE_BF16) for n in numels]
+        bc.bc_forecast(h, 0.8, [o.data_ptr() for o in ref], bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        sets = [[empty_out(n, bc.DTYPE_BF16) for n in numels] for _ in range(8)]
+        st0 = bc.bc_cache_stats(h)
+        torch.cuda._sleep(100_000_000)            # device time ahead of the queued uploads
+        for outs in sets:
+            bc.bc_forecast(h, 0.8, [o.data_ptr() for o in outs], bc.DTYPE_BF16, stream())
+        torch.cuda.synchronize()
+        assert bc.bc_cache_stats(h)["table_uploads"] - st0["table_uploads"] == 8
+        for outs in sets:
+            for a, b in zip(ref, outs):
+                assert torch.equal(a, b)
+        bc.bc_cache_check(h)
+    finally:
+        bc.bc_cache_destroy(h)
+
+
 @pytest.mark.parametrize("kernel", KERNELS, ids=KNAME.get)
 def test_many_layers_on_two_streams_share_the_device_table(kernel):
     # Forecasts over more layers than a parameter block holds read the handle's one device
